@@ -1,0 +1,239 @@
+"""Literal CPU oracle of the batched schedulers (A_max, A_min, H-SF).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this module.  The CUDA path shares no code with it.
+
+This is the slowest, most literal reading of the paper: it keeps the waiting set R_t and the active
+set S_t as explicit Python lists, and checks the future-memory constraint at *every* step t' from t
+to the last projected step (no endpoint shortcut).  Pure Python loops: small instances only.
+
+Model (Section 2, "Batch Processing, Memory Constraint, and Cancellation of Requests"):
+one worker with a KV cache of M tokens; a batch takes one unit of time; every member of the batch
+generates one output token; a job's memory is its prompt size plus the tokens generated so far
+(eq. constraintM); cancelling a job discards its tokens and returns it to the waiting set, its true
+output length o_i unchanged.  TEL = sum over jobs of (completion step - arrival step) (eq. latency;
+with all arrivals at 0 this is the paper's L_i = t + o_i of a job whose final start is t).
+
+Readings of the text that this oracle fixes (each is also listed in the design notes):
+
+* Memory timing ("W reading").  Step t processes batch B_t; each member's token count g goes up by
+  one; the memory of step t is  sum_{i in B_t} (s_i + g_i)  with g taken after the step, and must
+  be <= M.  A job started at step p with length L occupies steps p..p+L-1 (memory s+1 .. s+L) and
+  completes at C = p + L.  Completed jobs free their memory before the next step.  This is eq.
+  constraintM evaluated at the end of each batch.  It accepts both schedules I_1 and I_2 of the
+  example after Definition 1 and makes I_3 optimal there (TEL 12), and reproduces Example 1.
+* Future feasibility (eq. Constraint).  A candidate set U started at t is feasible with the active
+  set S' iff for every step t' >= t:
+      sum_{j in S' u U, t' <= e_j} (s_j + (t' - p_j) + 1) <= M,
+  where p_j is the job's (last) start (t for members of U) and e_j = p_j + Lhat_j - 1 its last
+  projected step.  Lhat is the policy's length estimate: o (H-SF, Section 3.1), u (A_max,
+  Algorithm malb) or the running lower bound õ (A_min, Algorithm milb).  For an active A_min job
+  that has already passed its estimate, e_j = max(p_j + õ_j - 1, t): it is known to be unfinished,
+  so it is projected for at least the current step.  The check covers every t' >= t (as stated
+  for A_max and H-SF), so if S' alone fails at some future step nothing is admitted.
+* Admission order.  The eligible waiting set (arrived, not active, not done) is sorted by
+  (key, request index) with key = u (A_max), õ (A_min) or o (H-SF); the policy admits the largest
+  feasible *prefix* ("in order", Algorithm milb).  The papers' "break ties uniformly at random"
+  becomes "smaller request index first"; the workload generator makes index order random.
+* A_min eviction (Algorithm milb / milbrevise).  If sum_{i in S_t} (s_i + g_i + 1) > M, sort S_t by
+  (õ_i, index) ascending and remove jobs one at a time until the rest fits.  Each removed job:
+  eviction count + 1, õ_i <- max(õ_i, g_i) (the refinement never lowers a certified lower bound),
+  g_i <- 0, back to the waiting set, and eligible in the same step's admission ("unprocessed or
+  restartable requests", Section 4).  Both the max and the same-step eligibility are switchable
+  for sensitivity studies (``refine`` / ``same_step``).
+* Arrivals (an extension: the paper has all a_i = 0).  Request i is eligible from step a_i on;
+  when nothing is active or eligible, time jumps to the next arrival.  Makespan = max C_i.
+* Step cap.  A run that has processed ``step_cap`` batches without finishing stops with status
+  STEPCAP.  Default cap: 64 * (n + sum_i o_i).
+"""
+from __future__ import annotations
+
+from typing import Sequence
+
+AMAX, AMIN, HSF = 0, 1, 2
+POLICY_NAMES = {AMAX: "A_max", AMIN: "A_min", HSF: "H-SF"}
+
+OK, E_INVAL, E_INFEASIBLE, E_STEPCAP = 0, -1, -2, -3
+
+_WAITING, _ACTIVE, _DONE = 0, 1, 2
+
+
+def default_step_cap(o: Sequence[int]) -> int:
+    return 64 * (len(o) + sum(int(x) for x in o))
+
+
+def validate(policy: int, M: int, a, s, l, u, o) -> int:
+    """Per-instance input check: 1 <= l <= o <= u, s >= 1, a >= 0, s + o <= M (s + u <= M for A_max)."""
+    for i in range(len(o)):
+        if s[i] < 1 or a[i] < 0 or l[i] < 1 or l[i] > o[i] or o[i] > u[i]:
+            return E_INVAL
+    for i in range(len(o)):
+        if s[i] + o[i] > M:
+            return E_INFEASIBLE
+        if policy == AMAX and s[i] + u[i] > M:
+            return E_INFEASIBLE
+    return OK
+
+
+def _empty_result(status: int, n: int) -> dict:
+    return dict(total_latency=0, makespan=0, peak_memory=0, evictions=0, steps=0,
+                request_steps=0, status=status, completion=[0] * n)
+
+
+def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
+             refine: str = "max", same_step: bool = True, trace: list | None = None) -> dict:
+    """Run one instance; return the result record plus per-request completion steps.
+
+    ``trace`` (optional list) receives one dict per processed step: t, the batch, the admitted
+    and the evicted request indices, and the step's memory.
+    """
+    n = len(o)
+    a = [int(x) for x in a]
+    s = [int(x) for x in s]
+    l = [int(x) for x in l]
+    u = [int(x) for x in u]
+    o = [int(x) for x in o]
+    st = validate(policy, M, a, s, l, u, o)
+    if st != OK:
+        return _empty_result(st, n)
+    if n == 0:
+        return _empty_result(OK, 0)
+    cap = default_step_cap(o) if step_cap is None else int(step_cap)
+
+    state = [_WAITING] * n
+    start = [None] * n  # last start p_i
+    gen = [0] * n  # tokens generated since the last start, g_i
+    otil = list(l)  # õ_i, the running lower bound (A_min)
+    completion = [0] * n
+
+    tel = makespan = peak = evictions = steps = request_steps = 0
+    status = OK
+    t = min(a)
+    n_done = 0
+
+    def est_len(i: int) -> int:
+        if policy == HSF:
+            return o[i]
+        if policy == AMAX:
+            return u[i]
+        return otil[i]
+
+    def key(i: int) -> int:
+        return est_len(i)  # the sort key is the length estimate for all three policies
+
+    def feasible(active: list, new: list) -> bool:
+        """eq. Constraint at every step t' from t to the last projected step (literal)."""
+        jobs = []  # (start, last projected step, prompt)
+        for j in active:
+            e = start[j] + est_len(j) - 1
+            if policy == AMIN:
+                e = max(e, t)
+            jobs.append((start[j], e, s[j]))
+        for j in new:
+            jobs.append((t, t + est_len(j) - 1, s[j]))
+        if not jobs:
+            return True
+        horizon = max(e for _, e, _ in jobs)
+        for tp in range(t, horizon + 1):
+            total = 0
+            for p, e, sj in jobs:
+                if tp <= e:
+                    total += sj + (tp - p) + 1
+            if total > M:
+                return False
+        return True
+
+    while n_done < n:
+        if steps >= cap:
+            status = E_STEPCAP
+            break
+        waiting = [i for i in range(n) if state[i] == _WAITING and a[i] <= t]
+        active = [i for i in range(n) if state[i] == _ACTIVE]
+        if not waiting and not active:
+            t = min(a[i] for i in range(n) if state[i] == _WAITING)
+            continue
+
+        evicted = []
+        if policy == AMIN:
+            need = sum(s[i] + gen[i] + 1 for i in active)
+            if need > M:
+                order = sorted(active, key=lambda i: (otil[i], i))
+                for i in order:
+                    if need <= M:
+                        break
+                    need -= s[i] + gen[i] + 1
+                    new_bound = max(otil[i], gen[i]) if refine == "max" else gen[i]
+                    assert new_bound >= otil[i] or refine != "max"
+                    otil[i] = new_bound
+                    gen[i] = 0
+                    start[i] = None
+                    state[i] = _WAITING
+                    evictions += 1
+                    evicted.append(i)
+                active = [i for i in active if state[i] == _ACTIVE]
+                if same_step:
+                    waiting = waiting + evicted
+                    waiting = [i for i in range(n) if i in set(waiting)]
+
+        waiting.sort(key=lambda i: (key(i), i))
+        admitted = []
+        for i in waiting:
+            if feasible(active, admitted + [i]):
+                admitted.append(i)
+            else:
+                break
+        for i in admitted:
+            state[i] = _ACTIVE
+            start[i] = t
+            gen[i] = 0
+
+        batch = active + admitted
+        for i in batch:
+            gen[i] += 1
+        mem = sum(s[i] + gen[i] for i in batch)
+        assert mem <= M, (t, mem, M)
+        peak = max(peak, mem)
+        request_steps += len(batch)
+        steps += 1
+        finished = []
+        for i in batch:
+            if gen[i] == o[i]:
+                state[i] = _DONE
+                completion[i] = t + 1
+                tel += t + 1 - a[i]
+                makespan = max(makespan, t + 1)
+                n_done += 1
+                finished.append(i)
+                assert completion[i] - start[i] == o[i]
+        if policy == AMIN:
+            for i in batch:
+                assert otil[i] <= o[i]
+        if trace is not None:
+            trace.append(dict(t=t, batch=sorted(batch), admitted=list(admitted),
+                              evicted=list(evicted), finished=sorted(finished), mem=mem))
+        t += 1
+
+    return dict(total_latency=tel, makespan=makespan, peak_memory=peak, evictions=evictions,
+                steps=steps, request_steps=request_steps, status=status, completion=completion)
+
+
+def is_feasible_schedule(M: int, s: Sequence[int], o: Sequence[int], starts: Sequence[int]) -> bool:
+    """Check a non-preemptive schedule (job i runs steps starts[i] .. starts[i]+o[i]-1) against
+    eq. constraintM under the W reading: at every step the batch's memory sum (s_i + g_i), with g_i
+    counted after the step, is at most M."""
+    if not starts:
+        return True
+    end = max(p + oi for p, oi in zip(starts, o))
+    for tp in range(min(starts), end):
+        total = 0
+        for p, si, oi in zip(starts, s, o):
+            if p <= tp <= p + oi - 1:
+                total += si + (tp - p) + 1
+        if total > M:
+            return False
+    return True
+
+
+def schedule_tel(a: Sequence[int], o: Sequence[int], starts: Sequence[int]) -> int:
+    """TEL of a schedule given final starts (eq. latency): sum (p_i + o_i - a_i)."""
+    return sum(p + oi - ai for p, oi, ai in zip(starts, o, a))

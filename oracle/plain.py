@@ -1,0 +1,113 @@
+"""ctypes wrapper of the plain C oracle (``oracle/plain.c``).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this module.  It shares no code with the CUDA path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from pathlib import Path
+
+import numpy as np
+
+_HERE = Path(__file__).resolve().parent
+_SRC = _HERE / "plain.c"
+_SO = _HERE / "_build" / "liboracle.so"
+
+RESULT_DTYPE = np.dtype([
+    ("total_latency", "<i8"), ("makespan", "<i8"), ("peak_memory", "<i8"),
+    ("evictions", "<i8"), ("steps", "<i8"), ("request_steps", "<i8"),
+    ("status", "<i4"), ("pad", "<i4"),
+])
+FIELDS = ("total_latency", "makespan", "peak_memory", "evictions", "steps", "request_steps", "status")
+
+_lib = None
+
+
+def build(force: bool = False) -> Path:
+    """Compile the C oracle into oracle/_build/liboracle.so (plain gcc, -O2)."""
+    _SO.parent.mkdir(parents=True, exist_ok=True)
+    if force or not _SO.exists() or _SO.stat().st_mtime < _SRC.stat().st_mtime:
+        tmp = _SO.with_suffix(f".so.{os.getpid()}")
+        subprocess.run(["gcc", "-O2", "-std=c11", "-D_GNU_SOURCE", "-shared", "-fPIC", "-o", str(tmp),
+                        str(_SRC), "-lpthread"], check=True)
+        os.replace(tmp, _SO)
+    return _SO
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        L = ctypes.CDLL(str(_SO))
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        i64p = ctypes.POINTER(ctypes.c_int64)
+        L.oracle_run.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i32p, i32p, i32p, i32p,
+                                 i32p, ctypes.c_int64, ctypes.c_void_p, i64p]
+        L.oracle_run.restype = ctypes.c_int
+        L.oracle_run_batch.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i64p, i32p, i32p,
+                                       i32p, i32p, i32p, ctypes.c_int64, ctypes.c_void_p, i64p,
+                                       ctypes.c_int32]
+        L.oracle_run_batch.restype = ctypes.c_int
+        L.oracle_default_step_cap.argtypes = [ctypes.c_int32, i32p]
+        L.oracle_default_step_cap.restype = ctypes.c_int64
+        _lib = L
+    return _lib
+
+
+def _i32(x) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+
+
+def _p32(x: np.ndarray):
+    return x.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def _p64(x: np.ndarray | None):
+    if x is None:
+        return ctypes.POINTER(ctypes.c_int64)()
+    return x.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
+
+
+def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool = False) -> dict:
+    """One instance.  Returns the result fields (and 'completion' if asked)."""
+    a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
+    n = int(o.shape[0])
+    res = np.zeros(1, dtype=RESULT_DTYPE)
+    comp = np.zeros(max(n, 1), dtype=np.int64) if completions else None
+    lib().oracle_run(int(policy), int(M), n, _p32(a), _p32(s), _p32(l), _p32(u), _p32(o),
+                     int(step_cap), res.ctypes.data, _p64(comp))
+    out = {k: int(res[0][k]) for k in FIELDS}
+    if completions:
+        out["completion"] = comp[:n].tolist()
+    return out
+
+
+def run_batch(policy: int, M: int, offsets, a, s, l, u, o, step_cap: int = 0, n_threads: int = 1,
+              completions: bool = False):
+    """Many instances in CSR layout.  Returns a structured array (RESULT_DTYPE) and optionally the
+    per-request completion steps."""
+    offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
+    n_inst = int(offsets.shape[0] - 1)
+    res = np.zeros(n_inst, dtype=RESULT_DTYPE)
+    comp = np.zeros(max(int(offsets[-1]), 1), dtype=np.int64) if completions else None
+    lib().oracle_run_batch(int(policy), int(M), n_inst, _p64(offsets), _p32(a), _p32(s), _p32(l),
+                           _p32(u), _p32(o), int(step_cap), res.ctypes.data, _p64(comp),
+                           int(n_threads))
+    if completions:
+        return res, comp[: int(offsets[-1])]
+    return res
+
+
+def run_workload(policy: int, w, step_cap: int = 0, n_threads: int = 1, completions: bool = False):
+    """Convenience: run a ``Workload`` (from the seeded generator) through the C oracle."""
+    return run_batch(policy, w.M, w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o,
+                     step_cap=step_cap, n_threads=n_threads, completions=completions)
+
+
+def default_step_cap(o) -> int:
+    o = _i32(o)
+    return int(lib().oracle_default_step_cap(int(o.shape[0]), _p32(o)))

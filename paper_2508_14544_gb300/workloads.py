@@ -1,0 +1,228 @@
+"""Seeded synthetic request workloads for the batched scheduler simulator.
+
+This module only draws input arrays (arrival step, prompt size, predicted interval, true output
+length).  It holds none of the scheduling arithmetic, so both the CPU oracle (``oracle/``) and the
+CUDA path consume exactly the same arrays.
+
+The paper evaluates on 2,000 sampled LMSYS-Chat-1M conversations (Section 6, "Dataset Overview").
+That dataset is not available here; the five synthetic workloads below stand in for it.  Their
+shapes follow the problem model of Section 2: every request has a prompt size s_i, a hidden output
+length o_i and a predicted interval [l_i, u_i] containing o_i (Section 2, "Prediction Interval for
+Output Length"; per-request intervals as in Section 4.2 and Experiments 2-3 of Section 6).
+
+Interval rule (all workloads): alpha = a/b is a rational, l_i ~ U{ceil(alpha*o_i) .. o_i} and
+u_i = ceil(l_i / alpha).  Both ceilings are computed in integers,
+ceil(a*o/b) = (a*o + b - 1) // b and ceil(l*b/a) = (l*b + a - 1) // a, so l_i <= o_i <= u_i holds
+exactly (no float rounding).
+
+Per-instance seeding: instance i of a workload draws from ``numpy.random.default_rng(seed0 + i)``
+in the fixed order s, o, l, arrivals, so any subset of instances is reproducible on its own.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from fractions import Fraction
+from typing import Callable, Sequence
+
+import numpy as np
+
+__all__ = [
+    "Workload",
+    "WORKLOADS",
+    "make_workload",
+    "make_instance",
+    "interval_for",
+    "concat_instances",
+]
+
+
+@dataclass
+class Workload:
+    """A batch of independent scheduling instances in CSR layout (int32 SoA arrays)."""
+
+    name: str
+    M: int
+    offsets: np.ndarray  # int64 [n_instances + 1]
+    arrival: np.ndarray  # int32 [n_total]  a_i (step at which request i becomes eligible)
+    prompt: np.ndarray  # int32 [n_total]  s_i
+    lower: np.ndarray  # int32 [n_total]  l_i
+    upper: np.ndarray  # int32 [n_total]  u_i
+    true_o: np.ndarray  # int32 [n_total]  o_i
+    alpha: list = field(default_factory=list)  # per-instance Fraction
+    instance_ids: np.ndarray | None = None  # global instance id of each row
+
+    @property
+    def n_instances(self) -> int:
+        return int(self.offsets.shape[0] - 1)
+
+    @property
+    def n_total(self) -> int:
+        return int(self.offsets[-1])
+
+    def instance(self, i: int) -> dict:
+        lo, hi = int(self.offsets[i]), int(self.offsets[i + 1])
+        return dict(
+            M=self.M,
+            a=self.arrival[lo:hi],
+            s=self.prompt[lo:hi],
+            l=self.lower[lo:hi],
+            u=self.upper[lo:hi],
+            o=self.true_o[lo:hi],
+        )
+
+    def uniform_n(self) -> int | None:
+        d = np.diff(self.offsets)
+        return int(d[0]) if d.size and np.all(d == d[0]) else None
+
+    def subset(self, rows: Sequence[int]) -> "Workload":
+        parts = [self.instance(int(i)) for i in rows]
+        ids = None if self.instance_ids is None else self.instance_ids[np.asarray(rows, dtype=np.int64)]
+        return concat_instances(self.name, self.M, parts, [self.alpha[int(i)] for i in rows], ids)
+
+
+def interval_for(o: np.ndarray, alpha: Fraction, rng: np.random.Generator) -> tuple[np.ndarray, np.ndarray]:
+    """Draw l ~ U{ceil(alpha*o)..o} and set u = ceil(l/alpha), in exact integer arithmetic."""
+    a, b = alpha.numerator, alpha.denominator
+    o64 = o.astype(np.int64)
+    lo = (a * o64 + b - 1) // b
+    lo = np.maximum(lo, 1)
+    l = rng.integers(lo, o64 + 1)  # inclusive upper bound via +1
+    u = (l * b + a - 1) // a
+    return l.astype(np.int32), u.astype(np.int32)
+
+
+def _poisson_arrivals(n: int, rate: float, rng: np.random.Generator) -> np.ndarray:
+    gaps = rng.exponential(scale=1.0 / rate, size=n)
+    return np.floor(np.cumsum(gaps)).astype(np.int64).astype(np.int32)
+
+
+# --- per-workload instance recipes -------------------------------------------------------------
+
+
+def _c1(i: int, rng: np.random.Generator):
+    n = 50
+    s = rng.integers(1, 21, size=n)
+    o = rng.integers(1, 101, size=n)
+    alpha = Fraction(1, 2)
+    l, u = interval_for(o, alpha, rng)
+    return np.zeros(n, np.int32), s, o, l, u, alpha
+
+
+_C2_ALPHAS = (Fraction(1, 5), Fraction(1, 2), Fraction(4, 5), Fraction(1, 1))
+
+
+def _c2(i: int, rng: np.random.Generator):
+    n = 1000
+    s = rng.integers(1, 65, size=n)
+    o = rng.integers(1, 513, size=n)
+    alpha = _C2_ALPHAS[(i // 256) % 4]
+    l, u = interval_for(o, alpha, rng)
+    return np.zeros(n, np.int32), s, o, l, u, alpha
+
+
+def _c3(i: int, rng: np.random.Generator):
+    n = 10_000
+    s = np.clip(np.rint(rng.lognormal(mean=5.0, sigma=0.8, size=n)), 1, 4096).astype(np.int64)
+    o = np.clip(rng.geometric(p=1.0 / 300.0, size=n), 1, 4096).astype(np.int64)
+    alpha = Fraction(3, 5)
+    l, u = interval_for(o, alpha, rng)
+    a = _poisson_arrivals(n, 0.5, rng)
+    return a, s, o, l, u, alpha
+
+
+def _c4(i: int, rng: np.random.Generator):
+    n = 2000
+    s = rng.integers(16, 257, size=n)
+    short = rng.random(size=n) < 0.7
+    o = np.where(short, rng.integers(1, 33, size=n), rng.integers(512, 2049, size=n))
+    alpha = Fraction((i // 4096) % 10 + 1, 10)
+    l, u = interval_for(o, alpha, rng)
+    return np.zeros(n, np.int32), s, o, l, u, alpha
+
+
+def _c5(i: int, rng: np.random.Generator):
+    n = 100_000
+    s = rng.integers(1, 2049, size=n)
+    o = np.clip(rng.zipf(1.2, size=n), 1, 8192).astype(np.int64)
+    alpha = Fraction(3, 10)
+    l, u = interval_for(o, alpha, rng)
+    a = _poisson_arrivals(n, 2.0, rng)
+    return a, s, o, l, u, alpha
+
+
+@dataclass(frozen=True)
+class _Spec:
+    name: str
+    M: int
+    n_instances: int
+    seed0: int
+    recipe: Callable
+    description: str
+
+
+WORKLOADS: dict[str, _Spec] = {
+    "c1": _Spec("c1", 2000, 1, 0, _c1,
+                "1 instance, n=50 at t=0, M=2000, s~U{1..20}, o~U{1..100}, alpha=1/2, seed 0"),
+    "c2": _Spec("c2", 16384, 1024, 1_000_000, _c2,
+                "1024 instances x n=1000 at t=0, M=16384, s~U{1..64}, o~U{1..512}, "
+                "alpha in {1/5,1/2,4/5,1} (256 seeds each)"),
+    "c3": _Spec("c3", 65536, 256, 2_000_000, _c3,
+                "256 instances x n=10^4, Poisson arrivals rate 0.5/step, M=65536, "
+                "s=round(lognormal(5,0.8)) in [1,4096], o~Geom(1/300) in [1,4096], alpha=3/5"),
+    "c4": _Spec("c4", 32768, 40960, 3_000_000, _c4,
+                "alpha in {0.1..1.0} x 4096 seeds, n=2000 at t=0, M=32768, s~U{16..256}, "
+                "o: 70% U{1..32}, 30% U{512..2048}"),
+    "c5": _Spec("c5", 500_000, 64, 4_000_000, _c5,
+                "64 instances x n=10^5, Poisson arrivals rate 2/step, M=500000, s~U{1..2048}, "
+                "o~Zipf(1.2) in [1,8192], alpha=3/10"),
+}
+
+
+def make_instance(name: str, i: int) -> dict:
+    """One instance of a named workload as a dict of int32 arrays plus M and alpha."""
+    spec = WORKLOADS[name]
+    rng = np.random.default_rng(spec.seed0 + i)
+    a, s, o, l, u, alpha = spec.recipe(i, rng)
+    return dict(
+        M=spec.M,
+        a=np.asarray(a, np.int32),
+        s=np.asarray(s, np.int32),
+        o=np.asarray(o, np.int32),
+        l=np.asarray(l, np.int32),
+        u=np.asarray(u, np.int32),
+        alpha=alpha,
+    )
+
+
+def concat_instances(name: str, M: int, parts: list[dict], alphas: list | None = None,
+                     ids: np.ndarray | None = None) -> Workload:
+    sizes = np.array([len(p["o"]) for p in parts], dtype=np.int64)
+    offsets = np.zeros(len(parts) + 1, dtype=np.int64)
+    np.cumsum(sizes, out=offsets[1:])
+
+    def cat(k):
+        if not parts:
+            return np.zeros(0, np.int32)
+        return np.ascontiguousarray(np.concatenate([np.asarray(p[k], np.int32) for p in parts]))
+
+    return Workload(
+        name=name,
+        M=int(M),
+        offsets=offsets,
+        arrival=cat("a"),
+        prompt=cat("s"),
+        lower=cat("l"),
+        upper=cat("u"),
+        true_o=cat("o"),
+        alpha=list(alphas) if alphas is not None else [p.get("alpha") for p in parts],
+        instance_ids=ids,
+    )
+
+
+def make_workload(name: str, instances: Sequence[int] | range | None = None) -> Workload:
+    """Generate a named workload (all instances, or the listed instance ids)."""
+    spec = WORKLOADS[name]
+    ids = range(spec.n_instances) if instances is None else instances
+    ids = np.asarray(list(ids), dtype=np.int64)
+    parts = [make_instance(name, int(i)) for i in ids]
+    return concat_instances(name, spec.M, parts, [p["alpha"] for p in parts], ids)

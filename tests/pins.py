@@ -1,0 +1,108 @@
+"""Checks of an oracle implementation against values the paper and the mathematics fix.
+
+``check_all(sim)`` runs every pin against ``sim(policy, M, a, s, l, u, o) -> dict`` (a dict with
+the result fields and 'completion') and returns the list of failures.  The pin tests call it on
+both oracles; the mutation tests call it on deliberately broken copies of the literal oracle and
+expect failures.
+"""
+from __future__ import annotations
+
+import json
+from pathlib import Path
+
+GOLDEN = Path(__file__).resolve().parent / "golden"
+AMAX, AMIN, HSF = 0, 1, 2
+POL = {"AMAX": AMAX, "AMIN": AMIN, "HSF": HSF}
+FIELDS = ("total_latency", "makespan", "peak_memory", "evictions", "steps", "request_steps")
+
+
+def load(name: str) -> dict:
+    return json.loads((GOLDEN / name).read_text())
+
+
+def wave_cases():
+    """Identical jobs with exact intervals (l = u = o), n = k*W, M in [k(s+o), k(s+o)+s]:
+    nothing can start while a wave runs (a job started d steps into a wave would need
+    s + o - d more tokens of room at the wave's last step, and the slack is at most s < s+o-d),
+    so the jobs run in W waves of k, each lasting o steps.  Closed form from the model of
+    Section 2: TEL = k*o*W(W+1)/2, makespan W*o, peak k(s+o), steps W*o, request steps n*o."""
+    out = []
+    for (k, W, s, o, r) in [(1, 3, 1, 1, 0), (2, 3, 1, 4, 1), (3, 4, 2, 5, 2), (5, 2, 3, 2, 0),
+                            (4, 5, 1, 3, 1), (2, 6, 4, 1, 3), (7, 3, 2, 6, 2)]:
+        n = k * W
+        M = k * (s + o) + r
+        exp = dict(total_latency=k * o * W * (W + 1) // 2, makespan=W * o, peak_memory=k * (s + o),
+                   evictions=0, steps=W * o, request_steps=n * o)
+        out.append(((k, W, s, o, r), M, [0] * n, [s] * n, [o] * n, [o] * n, [o] * n, exp))
+    return out
+
+
+def amax_wave_cases():
+    """A_max on identical jobs whose true length o is below the upper bound u, M = k(s+u):
+    A_max projects every job to u, so it starts k jobs at a time and nothing else fits until
+    the wave completes (after o steps) -- Example 1 generalised.  TEL = sum over waves w of
+    |wave_w| * (w+1) * o, with waves of k and a last partial wave."""
+    out = []
+    for (k, n, s, o, u) in [(2, 5, 1, 1, 4), (3, 7, 2, 2, 5), (1, 4, 3, 3, 3), (4, 9, 1, 2, 9)]:
+        M = k * (s + u)
+        tel, w, left = 0, 0, n
+        while left > 0:
+            m = min(k, left)
+            tel += m * (w + 1) * o
+            left -= m
+            w += 1
+        exp = dict(total_latency=tel, makespan=w * o, evictions=0, steps=w * o, request_steps=n * o,
+                   peak_memory=min(k, n) * (s + o))
+        out.append(((k, n, s, o, u), M, [0] * n, [s] * n, [o] * n, [u] * n, [o] * n, exp))
+    return out
+
+
+def check_all(sim) -> list:
+    fails = []
+
+    def chk(tag, got, exp):
+        for key, val in exp.items():
+            if key == "completion_sorted":
+                if sorted(got["completion"]) != val:
+                    fails.append((tag, key, sorted(got["completion"]), val))
+            elif key == "starts":
+                continue
+            elif got.get(key) != val:
+                fails.append((tag, key, got.get(key), val))
+
+    def run(tag, *args):
+        try:
+            return sim(*args)
+        except AssertionError as e:  # an internal invariant tripped
+            fails.append((tag, "assertion", str(e), None))
+            return None
+
+    pe = load("paper_examples.json")
+    ex = pe["example1"]
+    for pname, exp in ex["expect"].items():
+        r = run("example1/" + pname, POL[pname], ex["M"], ex["a"], ex["s"], ex["l"], ex["u"], ex["o"])
+        if r is not None:
+            chk("example1/" + pname, r, exp)
+    d1 = pe["def1_example"]
+    r = run("def1/HSF", HSF, d1["M"], d1["a"], d1["s"], d1["o"], d1["o"], d1["o"])
+    if r is not None:
+        chk("def1/HSF", r, d1["expect"]["HSF"])
+
+    ht = load("hand_traces.json")
+    for name, case in ht.items():
+        if name.startswith("_"):
+            continue
+        r = run(name, POL[case["policy"]], case["M"], case["a"], case["s"], case["l"], case["u"], case["o"])
+        if r is not None:
+            chk(name, r, case["expect"])
+
+    for tag, M, a, s, l, u, o, exp in wave_cases():
+        for p in (AMAX, AMIN, HSF):
+            r = run(f"waves{tag}/{p}", p, M, a, s, l, u, o)
+            if r is not None:
+                chk(f"waves{tag}/{p}", r, exp)
+    for tag, M, a, s, l, u, o, exp in amax_wave_cases():
+        r = run(f"amaxwaves{tag}", AMAX, M, a, s, l, u, o)
+        if r is not None:
+            chk(f"amaxwaves{tag}", r, exp)
+    return fails
