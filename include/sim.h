@@ -1,0 +1,163 @@
+/*
+ * sim.h - C ABI of the batched scheduler simulator (libsim.so, CUDA, sm_103a).
+ *
+ * The library simulates many independent instances of the single-worker LLM-inference
+ * scheduling problem of arXiv 2508.14544 ("Adaptively Robust LLM Inference Optimization under
+ * Prediction Uncertainty") on one GPU, under one of three policies:
+ *
+ *   SIM_AMAX - A_max, Algorithm malb (Section 3.2): every output length is taken to be its
+ *              predicted upper bound u_i; each step admits the largest prefix of the waiting set,
+ *              sorted by (u_i, request index), that keeps the projected memory within M at every
+ *              future step (eq. Constraint).  Never cancels a job.
+ *   SIM_AMIN - A_min, Algorithms milb and milbrevise (Section 4, 4.2): each request starts with the
+ *              lower bound l_i as its length estimate; when the next step would exceed M, active
+ *              jobs are cancelled in ascending (estimate, index) order until the rest fits, and each
+ *              cancelled job's estimate becomes max(estimate, tokens generated); the waiting set is
+ *              then admitted as for A_max, using the estimates.
+ *   SIM_HSF  - the hindsight shortest-first benchmark H-SF, Algorithm off (Section 3.1, Appendix
+ *              B): like A_max with the true output lengths.
+ *
+ * Model (Section 2): a worker with a KV cache of M tokens runs one batch per unit of time; every
+ * member generates one token; a job's memory is its prompt size s_i plus the tokens generated so
+ * far, and the memory of each step (counted after the step's tokens) must not exceed M
+ * (eq. constraintM).  Request i becomes eligible at step a_i (the paper has a_i = 0; arrivals are
+ * an extension); its completion step C_i is one past the step that generated its last token.
+ *
+ * Ties that the paper breaks "uniformly at random" are broken by the smaller request index
+ * (0-based position within the instance).  Outputs are deterministic and bit-identical to the CPU
+ * reference of the same rules.
+ *
+ * Threading: a context must not be used from two threads at once.  Different contexts are
+ * independent.  All calls act on the CUDA device that is current on the calling thread.
+ */
+#ifndef SIM_H_
+#define SIM_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { SIM_AMAX = 0, SIM_AMIN = 1, SIM_HSF = 2 } sim_policy;
+
+typedef enum {
+    SIM_OK = 0,
+    SIM_E_INVAL = -1,      /* bad argument, or an instance with l > o, o > u, l < 1, s < 1, a < 0 */
+    SIM_E_INFEASIBLE = -2, /* an instance has a request with s + o > M (or s + u > M under A_max) */
+    SIM_E_STEPCAP = -3,    /* an instance processed step_cap batches without finishing */
+    SIM_E_CUDA = -4,       /* a CUDA runtime call failed; see sim_last_error */
+    SIM_E_STATE = -5,      /* call out of order (e.g. sim_run before sim_load), or an internal check failed */
+    SIM_E_NOMEM = -6       /* host or device allocation failed */
+} sim_status;
+
+/* Per-instance result of sim_run (56 bytes). */
+typedef struct {
+    int64_t total_latency; /* TEL = sum_i (C_i - a_i)  (eq. latency) */
+    int64_t makespan;      /* max_i C_i */
+    int64_t peak_memory;   /* max over steps of the step's memory, sum over the batch of (s + tokens) */
+    int64_t evictions;     /* number of cancellations (always 0 for A_max and H-SF) */
+    int64_t steps;         /* batches processed (steps skipped while idle are not counted) */
+    int64_t request_steps; /* sum over steps of the batch size (tokens generated, wasted ones included) */
+    int32_t status;        /* sim_status of this instance */
+    int32_t _pad;
+} sim_result;
+
+typedef struct sim_ctx sim_ctx;
+
+/* Options for sim_set_option. */
+enum {
+    SIM_OPT_STEP_CAP = 1,           /* int64 > 0: stop an instance after this many batches
+                                       (status SIM_E_STEPCAP).  0 (default): 64 * (n + sum_i o_i). */
+    SIM_OPT_RECORD_COMPLETIONS = 2, /* 0/1: keep each request's completion step for
+                                       sim_get_completions (default 0). */
+    SIM_OPT_WARPS_PER_BLOCK = 3,    /* 1..8: simulation warps per thread block (default 4). */
+    SIM_OPT_SMEM_ACTIVE_CAP = 4     /* 32..4096, multiple of 32: active-set slots kept in shared
+                                       memory per instance (default 512).  Instances that need more
+                                       are re-run automatically with the active set in global
+                                       memory; results are identical. */
+};
+
+/*
+ * sim_create: set up a context for `n_instances` independent instances simulated under `policy`
+ * with KV-cache limit M tokens (Section 2).
+ *   policy      SIM_AMAX, SIM_AMIN or SIM_HSF.
+ *   M           1 <= M <= 2^26.
+ *   n_instances >= 1.
+ *   out         receives the new context (owned by the caller; free with sim_destroy).
+ * Touches no GPU memory.  Returns SIM_OK, SIM_E_INVAL or SIM_E_NOMEM.
+ */
+int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out);
+
+/*
+ * sim_load: load n_per_instance requests for every instance (uniform sizes).  Each array holds
+ * n_instances * n_per_instance int32 values, instance-major: request j of instance i is at
+ * [i * n_per_instance + j].
+ *   arrival_t  a_i >= 0: first step at which the request may be scheduled.
+ *   prompt_s   s_i >= 1: prompt size in tokens (Section 2; per-request as in Section 6).
+ *   lower_l    l_i: predicted lower bound of the output length, 1 <= l_i <= o_i.
+ *   upper_u    u_i: predicted upper bound, o_i <= u_i.
+ *   true_o     o_i >= 1: true output length (hidden from A_max and A_min; used by H-SF and by the
+ *              simulation itself to know when a job finishes).
+ *   device_ptrs 0: the arrays are host memory; 1: device memory on the current device.
+ * The library copies the data into device buffers it owns; the caller may free or reuse its
+ * arrays as soon as the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
+ * the call: they are reported in that instance's sim_result.status by sim_run.
+ * Returns SIM_OK, SIM_E_INVAL (n_per_instance < 0, null pointer), SIM_E_NOMEM or SIM_E_CUDA.
+ */
+int sim_load(sim_ctx *ctx, int32_t n_per_instance, const int32_t *arrival_t, const int32_t *prompt_s,
+             const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o, int device_ptrs);
+
+/*
+ * sim_load_csr: like sim_load with per-instance sizes.  `offsets` is HOST memory with
+ * n_instances + 1 non-decreasing int64 values, offsets[0] = 0; instance i owns requests
+ * [offsets[i], offsets[i+1]) of each array.  Empty instances are allowed (their result is all
+ * zeros with status SIM_OK).
+ */
+int sim_load_csr(sim_ctx *ctx, const int64_t *offsets, const int32_t *arrival_t, const int32_t *prompt_s,
+                 const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o, int device_ptrs);
+
+/*
+ * sim_run: simulate every loaded instance and write n_instances results to `out` (HOST memory).
+ *   cuda_stream  a cudaStream_t of the current device, or NULL for the default stream.
+ * Synchronous: returns after the results are in `out`.  Re-running without reloading gives
+ * identical results.  Returns the most negative per-instance status (SIM_OK if all succeeded),
+ * or SIM_E_STATE (nothing loaded), SIM_E_CUDA, SIM_E_NOMEM.
+ */
+int sim_run(sim_ctx *ctx, sim_result *out, void *cuda_stream);
+
+/*
+ * sim_get_completions: copy every request's completion step C_i of the last sim_run into
+ * `completion_t` (HOST, n_total int64, same layout as the loaded arrays; 0 for instances that did
+ * not run).  Requires SIM_OPT_RECORD_COMPLETIONS = 1 before sim_run; otherwise SIM_E_STATE.
+ */
+int sim_get_completions(sim_ctx *ctx, int64_t *completion_t);
+
+/*
+ * sim_competitive_ratio: per-instance ratio TEL(policy) / TEL(H-SF) (Definition cr, Section 3.1)
+ * of two contexts that ran the same instances, computed on the device in IEEE double.
+ *   ctx_policy, ctx_hsf  contexts after sim_run with equal n_instances (ctx_hsf under SIM_HSF).
+ *   cr_out               HOST, n_instances doubles; NaN where either instance failed or TEL(H-SF)=0.
+ * Returns SIM_OK, SIM_E_INVAL or SIM_E_STATE.
+ */
+int sim_competitive_ratio(const sim_ctx *ctx_policy, const sim_ctx *ctx_hsf, double *cr_out, void *cuda_stream);
+
+/* sim_kernel_launches: number of CUDA kernels this context has launched since sim_create
+ * (staging, simulation, fallback and ratio kernels).  ctx NULL -> -1. */
+int64_t sim_kernel_launches(const sim_ctx *ctx);
+
+/* sim_set_option: set one of the SIM_OPT_* options.  Returns SIM_OK or SIM_E_INVAL. */
+int sim_set_option(sim_ctx *ctx, int key, int64_t value);
+
+/* sim_last_error: NUL-terminated message of the last failing call on ctx ("" if none).  The
+ * pointer stays valid until the next call on ctx.  ctx may be NULL (message of the last sim_create). */
+const char *sim_last_error(const sim_ctx *ctx);
+
+/* sim_destroy: free the context and every device buffer it owns.  NULL is allowed. */
+void sim_destroy(sim_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SIM_H_ */

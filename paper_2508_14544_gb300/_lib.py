@@ -1,0 +1,145 @@
+"""ctypes binding of libsim.so (include/sim.h).
+
+Argument marshalling only: every step of the simulation runs in the library's CUDA kernels.
+There is no CPU fallback; if the library is missing or fails to load, ``lib()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from pathlib import Path
+
+import numpy as np
+
+from .build import LIB
+
+SIM_AMAX, SIM_AMIN, SIM_HSF = 0, 1, 2
+SIM_OK, SIM_E_INVAL, SIM_E_INFEASIBLE, SIM_E_STEPCAP, SIM_E_CUDA, SIM_E_STATE, SIM_E_NOMEM = 0, -1, -2, -3, -4, -5, -6
+SIM_OPT_STEP_CAP, SIM_OPT_RECORD_COMPLETIONS, SIM_OPT_WARPS_PER_BLOCK, SIM_OPT_SMEM_ACTIVE_CAP = 1, 2, 3, 4
+
+STATUS_NAMES = {0: "SIM_OK", -1: "SIM_E_INVAL", -2: "SIM_E_INFEASIBLE", -3: "SIM_E_STEPCAP", -4: "SIM_E_CUDA",
+                -5: "SIM_E_STATE", -6: "SIM_E_NOMEM"}
+
+
+class sim_result(ctypes.Structure):
+    _fields_ = [("total_latency", ctypes.c_int64), ("makespan", ctypes.c_int64), ("peak_memory", ctypes.c_int64),
+                ("evictions", ctypes.c_int64), ("steps", ctypes.c_int64), ("request_steps", ctypes.c_int64),
+                ("status", ctypes.c_int32), ("_pad", ctypes.c_int32)]
+
+
+RESULT_DTYPE = np.dtype([
+    ("total_latency", "<i8"), ("makespan", "<i8"), ("peak_memory", "<i8"), ("evictions", "<i8"),
+    ("steps", "<i8"), ("request_steps", "<i8"), ("status", "<i4"), ("_pad", "<i4"),
+])
+assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
+
+EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
+           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches")
+
+_lib = None
+
+
+class SimError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+def lib_path() -> Path:
+    p = os.environ.get("SIMGB_LIB")
+    return Path(p) if p else LIB
+
+
+def lib() -> ctypes.CDLL:
+    """Load libsim.so (it must have been built, e.g. by __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = lib_path()
+    if not path.exists():
+        raise RuntimeError(f"libsim.so not found at {path}: build it first (python -m paper_2508_14544_gb300.build)")
+    L = ctypes.CDLL(str(path))
+    vp, i32p, i64p = ctypes.c_void_p, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int64)
+    L.sim_create.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(vp)]
+    L.sim_create.restype = ctypes.c_int
+    L.sim_load.argtypes = [vp, ctypes.c_int32, vp, vp, vp, vp, vp, ctypes.c_int]
+    L.sim_load.restype = ctypes.c_int
+    L.sim_load_csr.argtypes = [vp, vp, vp, vp, vp, vp, vp, ctypes.c_int]
+    L.sim_load_csr.restype = ctypes.c_int
+    L.sim_run.argtypes = [vp, vp, vp]
+    L.sim_run.restype = ctypes.c_int
+    L.sim_get_completions.argtypes = [vp, vp]
+    L.sim_get_completions.restype = ctypes.c_int
+    L.sim_competitive_ratio.argtypes = [vp, vp, vp, vp]
+    L.sim_competitive_ratio.restype = ctypes.c_int
+    L.sim_set_option.argtypes = [vp, ctypes.c_int, ctypes.c_int64]
+    L.sim_set_option.restype = ctypes.c_int
+    L.sim_last_error.argtypes = [vp]
+    L.sim_last_error.restype = ctypes.c_char_p
+    L.sim_destroy.argtypes = [vp]
+    L.sim_destroy.restype = None
+    L.sim_kernel_launches.argtypes = [vp]
+    L.sim_kernel_launches.restype = ctypes.c_int64
+    _lib = L
+    return L
+
+
+# ---- thin wrappers with the C names -------------------------------------------------------------
+
+def sim_create(policy: int, M: int, n_instances: int) -> ctypes.c_void_p:
+    h = ctypes.c_void_p()
+    rc = lib().sim_create(int(policy), int(M), int(n_instances), ctypes.byref(h))
+    if rc != SIM_OK:
+        raise SimError(rc, sim_last_error(None))
+    return h
+
+
+def sim_last_error(ctx) -> str:
+    s = lib().sim_last_error(ctx)
+    return s.decode() if s else ""
+
+
+def sim_set_option(ctx, key: int, value: int) -> int:
+    return lib().sim_set_option(ctx, int(key), int(value))
+
+
+def _ptr(x) -> int:
+    """Address of a contiguous int32 host array or device tensor (torch)."""
+    if isinstance(x, np.ndarray):
+        return x.ctypes.data
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    raise TypeError(type(x))
+
+
+def sim_load(ctx, n_per_instance: int, a, s, l, u, o, device_ptrs: int) -> int:
+    return lib().sim_load(ctx, int(n_per_instance), _ptr(a), _ptr(s), _ptr(l), _ptr(u), _ptr(o), int(device_ptrs))
+
+
+def sim_load_csr(ctx, offsets: np.ndarray, a, s, l, u, o, device_ptrs: int) -> int:
+    assert offsets.dtype == np.int64 and offsets.flags.c_contiguous
+    return lib().sim_load_csr(ctx, offsets.ctypes.data, _ptr(a), _ptr(s), _ptr(l), _ptr(u), _ptr(o),
+                              int(device_ptrs))
+
+
+def sim_run(ctx, out: np.ndarray, stream: int = 0) -> int:
+    assert out.dtype == RESULT_DTYPE and out.flags.c_contiguous
+    return lib().sim_run(ctx, out.ctypes.data, ctypes.c_void_p(stream or None))
+
+
+def sim_get_completions(ctx, out: np.ndarray) -> int:
+    assert out.dtype == np.int64 and out.flags.c_contiguous
+    return lib().sim_get_completions(ctx, out.ctypes.data)
+
+
+def sim_competitive_ratio(ctx_policy, ctx_hsf, out: np.ndarray, stream: int = 0) -> int:
+    assert out.dtype == np.float64 and out.flags.c_contiguous
+    return lib().sim_competitive_ratio(ctx_policy, ctx_hsf, out.ctypes.data, ctypes.c_void_p(stream or None))
+
+
+def sim_kernel_launches(ctx) -> int:
+    return int(lib().sim_kernel_launches(ctx))
+
+
+def sim_destroy(ctx) -> None:
+    lib().sim_destroy(ctx)

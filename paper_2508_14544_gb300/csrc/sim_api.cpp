@@ -1,0 +1,434 @@
+// C ABI of the batched scheduler simulator (declared in include/sim.h).
+//
+// Host side only: argument checks, device buffers owned by the context, launches of the staging
+// and simulation kernels (sim_kernels.cu), and the capacity fallback (instances whose active set
+// outgrows the shared-memory workspace are re-run with a global-memory workspace).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "sim.h"
+#include "sim_internal.h"
+
+using simgb::DevResult;
+using simgb::InstInfo;
+using simgb::QEnt;
+
+struct sim_ctx {
+    int policy = 0;
+    int64_t M = 0;
+    int32_t n_inst = 0;
+    // options
+    int64_t step_cap = 0;
+    int record_completions = 0;
+    int wpb = 4;
+    int smem_ca = 512;
+    int dcap = 256;
+    // state
+    int device = -1;
+    bool loaded = false;
+    bool ran = false;
+    bool comp_valid = false;
+    int64_t n_total = 0;
+    int32_t n_max = 0;
+    // device buffers
+    int64_t *d_off = nullptr;
+    int32_t *d_raw = nullptr;  // 5 * cap_total
+    int64_t cap_total = 0;
+    QEnt *d_rec = nullptr;
+    int32_t *d_rec_a = nullptr;
+    InstInfo *d_info = nullptr;
+    DevResult *d_res = nullptr;
+    int64_t *d_comp = nullptr;
+    int32_t *d_counter = nullptr;
+    int32_t *d_work = nullptr;
+    unsigned char *d_gws = nullptr;
+    size_t gws_bytes = 0;
+    QEnt *d_main = nullptr;
+    size_t main_bytes = 0;
+    double *d_cr = nullptr;
+    int64_t launches = 0;
+    std::vector<DevResult> h_res;
+    std::string err;
+};
+
+static_assert(sizeof(sim_result) == 56, "sim_result must be 56 bytes");
+static_assert(sizeof(DevResult) == sizeof(sim_result), "device result layout");
+
+namespace {
+
+thread_local std::string g_create_err;
+
+int fail(sim_ctx *c, int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    if (c) c->err = buf; else g_create_err = buf;
+    return code;
+}
+
+int cuda_fail(sim_ctx *c, cudaError_t e, const char *what) {
+    return fail(c, SIM_E_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+template <typename T>
+void dfree(T *&p) {
+    if (p) cudaFree(p);
+    p = nullptr;
+}
+
+template <typename T>
+cudaError_t dalloc(T *&p, size_t bytes) {
+    dfree(p);
+    if (bytes == 0) bytes = 16;
+    void *q = nullptr;
+    cudaError_t e = cudaMalloc(&q, bytes);
+    if (e == cudaSuccess) p = static_cast<T *>(q);
+    return e;
+}
+
+int check_device(sim_ctx *c) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(c, e, "cudaGetDevice");
+    if (c->device >= 0 && dev != c->device)
+        return fail(c, SIM_E_STATE, "current device %d differs from the device %d the data was loaded on", dev,
+                    c->device);
+    c->device = dev;
+    return SIM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out) {
+    if (!out) return fail(nullptr, SIM_E_INVAL, "sim_create: out is NULL");
+    *out = nullptr;
+    if (policy < SIM_AMAX || policy > SIM_HSF) return fail(nullptr, SIM_E_INVAL, "sim_create: bad policy %d", policy);
+    if (M < 1 || M > simgb::kMaxM)
+        return fail(nullptr, SIM_E_INVAL, "sim_create: M=%lld outside [1, 2^26]", (long long)M);
+    if (n_instances < 1) return fail(nullptr, SIM_E_INVAL, "sim_create: n_instances=%d < 1", n_instances);
+    sim_ctx *c = new (std::nothrow) sim_ctx();
+    if (!c) return fail(nullptr, SIM_E_NOMEM, "sim_create: out of host memory");
+    c->policy = policy;
+    c->M = M;
+    c->n_inst = n_instances;
+    g_create_err.clear();
+    *out = c;
+    return SIM_OK;
+}
+
+int sim_set_option(sim_ctx *c, int key, int64_t value) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    switch (key) {
+        case SIM_OPT_STEP_CAP:
+            if (value < 0) return fail(c, SIM_E_INVAL, "STEP_CAP must be >= 0");
+            c->step_cap = value;
+            if (c->loaded) c->loaded = false;  // the cap is staged with the data: reload required
+            return SIM_OK;
+        case SIM_OPT_RECORD_COMPLETIONS:
+            c->record_completions = value ? 1 : 0;
+            return SIM_OK;
+        case SIM_OPT_WARPS_PER_BLOCK:
+            if (value < 1 || value > 8) return fail(c, SIM_E_INVAL, "WARPS_PER_BLOCK must be in [1, 8]");
+            c->wpb = int(value);
+            return SIM_OK;
+        case SIM_OPT_SMEM_ACTIVE_CAP:
+            if (value < 32 || value > 4096 || value % 32)
+                return fail(c, SIM_E_INVAL, "SMEM_ACTIVE_CAP must be a multiple of 32 in [32, 4096]");
+            c->smem_ca = int(value);
+            return SIM_OK;
+        default:
+            return fail(c, SIM_E_INVAL, "unknown option %d", key);
+    }
+}
+
+int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int32_t *s, const int32_t *l,
+                 const int32_t *u, const int32_t *o, int device_ptrs) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    c->loaded = false;
+    c->ran = false;
+    c->comp_valid = false;
+    if (!offsets) return fail(c, SIM_E_INVAL, "sim_load: offsets is NULL");
+    if (offsets[0] != 0) return fail(c, SIM_E_INVAL, "sim_load: offsets[0] must be 0");
+    int64_t n_max = 0;
+    for (int32_t i = 0; i < c->n_inst; ++i) {
+        const int64_t d = offsets[i + 1] - offsets[i];
+        if (d < 0) return fail(c, SIM_E_INVAL, "sim_load: offsets decrease at instance %d", i);
+        if (d > INT32_MAX / 2) return fail(c, SIM_E_INVAL, "sim_load: instance %d has too many requests", i);
+        n_max = std::max(n_max, d);
+    }
+    const int64_t nt = offsets[c->n_inst];
+    if (nt > 0 && (!a || !s || !l || !u || !o)) return fail(c, SIM_E_INVAL, "sim_load: NULL input array");
+    int rc = check_device(c);
+    if (rc) return rc;
+    cudaError_t e;
+    if (nt > c->cap_total || !c->d_raw) {
+        const int64_t cap = std::max<int64_t>(nt, 1);
+        if ((e = dalloc(c->d_raw, size_t(5) * cap * sizeof(int32_t))) != cudaSuccess ||
+            (e = dalloc(c->d_rec, size_t(cap) * sizeof(QEnt))) != cudaSuccess ||
+            (e = dalloc(c->d_rec_a, size_t(cap) * sizeof(int32_t))) != cudaSuccess) {
+            c->cap_total = 0;
+            return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_load: device allocation failed")
+                                                  : cuda_fail(c, e, "cudaMalloc");
+        }
+        dfree(c->d_comp);
+        c->cap_total = cap;
+    }
+    if (!c->d_off) {
+        if ((e = dalloc(c->d_off, size_t(c->n_inst + 1) * sizeof(int64_t))) != cudaSuccess ||
+            (e = dalloc(c->d_info, size_t(c->n_inst) * sizeof(InstInfo))) != cudaSuccess ||
+            (e = dalloc(c->d_res, size_t(c->n_inst) * sizeof(DevResult))) != cudaSuccess ||
+            (e = dalloc(c->d_counter, sizeof(int32_t) * 4)) != cudaSuccess ||
+            (e = dalloc(c->d_work, size_t(c->n_inst) * sizeof(int32_t))) != cudaSuccess)
+            return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_load: device allocation failed")
+                                                  : cuda_fail(c, e, "cudaMalloc");
+    }
+    const cudaMemcpyKind kind = device_ptrs ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    const int32_t *src[5] = {a, s, l, u, o};
+    for (int k = 0; k < 5; ++k) {
+        if (nt == 0) break;
+        e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t), kind, 0);
+        if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the input arrays");
+    }
+    e = cudaMemcpyAsync(c->d_off, offsets, size_t(c->n_inst + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, 0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the offsets");
+    simgb::StageParams sp;
+    sp.policy = c->policy;
+    sp.M = c->M;
+    sp.n_inst = c->n_inst;
+    sp.step_cap = c->step_cap;
+    sp.off = c->d_off;
+    sp.a = c->d_raw;
+    sp.s = c->d_raw + c->cap_total;
+    sp.l = c->d_raw + 2 * c->cap_total;
+    sp.u = c->d_raw + 3 * c->cap_total;
+    sp.o = c->d_raw + 4 * c->cap_total;
+    sp.rec = c->d_rec;
+    sp.rec_a = c->d_rec_a;
+    sp.info = c->d_info;
+    e = simgb::launch_stage(sp, 0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: staging kernel launch");
+    if (c->n_inst > 0) ++c->launches;
+    e = cudaStreamSynchronize(0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: staging kernel");
+    c->n_total = nt;
+    c->n_max = int32_t(n_max);
+    c->loaded = true;
+    return SIM_OK;
+}
+
+int sim_load(sim_ctx *c, int32_t n, const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+             const int32_t *o, int device_ptrs) {
+    if (!c) return SIM_E_INVAL;
+    if (n < 0) return fail(c, SIM_E_INVAL, "sim_load: n_per_instance=%d < 0", n);
+    std::vector<int64_t> off(size_t(c->n_inst) + 1);
+    for (int32_t i = 0; i <= c->n_inst; ++i) off[i] = int64_t(i) * n;
+    return sim_load_csr(c, off.data(), a, s, l, u, o, device_ptrs);
+}
+
+static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int32_t n_work, bool smem) {
+    cudaError_t e;
+    int dev = c->device;
+    int n_sm = 0, smem_optin = 0;
+    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    int wpb = c->wpb;
+    const int dcap = c->dcap;
+    int ca = smem ? c->smem_ca : ((std::max(c->n_max, 32) + 31) / 32) * 32;
+    size_t per_warp = simgb::warp_ws_bytes(ca, dcap);
+    size_t smem_bytes = 0;
+    if (smem) {
+        while (wpb > 1 && per_warp * wpb > size_t(smem_optin)) --wpb;
+        if (per_warp * wpb > size_t(smem_optin)) return fail(c, SIM_E_INVAL, "workspace does not fit shared memory");
+        smem_bytes = per_warp * wpb;
+        e = simgb::set_run_smem_limit(c->policy, smem_bytes);
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaFuncSetAttribute");
+    }
+    int per_sm = 1;
+    if (smem) {
+        int smem_sm = 0;
+        cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+        per_sm = std::max(1, int(size_t(smem_sm) / (smem_bytes + 1024)));
+        per_sm = std::min(per_sm, 64 / wpb);
+    } else {
+        per_sm = std::max(1, 16 / wpb);
+    }
+    int64_t blocks = int64_t(n_sm) * per_sm;
+    blocks = std::min<int64_t>(blocks, (n_work + wpb - 1) / wpb);
+    blocks = std::max<int64_t>(blocks, 1);
+    const int64_t slots = blocks * wpb;
+    const int64_t main_cap = std::max<int64_t>(c->n_max, 1);
+    const size_t main_need = size_t(slots) * 2 * main_cap * sizeof(QEnt);
+    if (main_need > c->main_bytes) {
+        if ((e = dalloc(c->d_main, main_need)) != cudaSuccess) {
+            c->main_bytes = 0;
+            return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_run: queue buffers") : cuda_fail(c, e, "cudaMalloc");
+        }
+        c->main_bytes = main_need;
+    }
+    if (!smem) {
+        const size_t need = size_t(slots) * per_warp;
+        if (need > c->gws_bytes) {
+            if ((e = dalloc(c->d_gws, need)) != cudaSuccess) {
+                c->gws_bytes = 0;
+                return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_run: workspace") : cuda_fail(c, e, "cudaMalloc");
+            }
+            c->gws_bytes = need;
+        }
+    }
+    simgb::RunParams p;
+    p.M = c->M;
+    p.n_work = n_work;
+    p.work = work_dev;
+    p.counter = c->d_counter;
+    p.rec = c->d_rec;
+    p.rec_a = c->d_rec_a;
+    p.info = c->d_info;
+    p.res = c->d_res;
+    p.completion = c->record_completions ? c->d_comp : nullptr;
+    p.ca = ca;
+    p.dcap = dcap;
+    p.use_smem = smem ? 1 : 0;
+    p.gws = c->d_gws;
+    p.gws_stride = int64_t(per_warp);
+    p.mainbuf = c->d_main;
+    p.main_cap = main_cap;
+    if ((e = cudaMemsetAsync(c->d_counter, 0, sizeof(int32_t), st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaMemsetAsync");
+    e = simgb::launch_run(c->policy, p, int(blocks), wpb, smem_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: kernel launch");
+    ++c->launches;
+    return SIM_OK;
+}
+
+int sim_run(sim_ctx *c, sim_result *out, void *stream) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    if (!c->loaded) return fail(c, SIM_E_STATE, "sim_run: nothing loaded (call sim_load first)");
+    if (!out) return fail(c, SIM_E_INVAL, "sim_run: out is NULL");
+    int rc = check_device(c);
+    if (rc) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if (c->record_completions) {
+        if (!c->d_comp && (e = dalloc(c->d_comp, size_t(c->cap_total) * sizeof(int64_t))) != cudaSuccess)
+            return fail(c, SIM_E_NOMEM, "sim_run: completion buffer");
+        if ((e = cudaMemsetAsync(c->d_comp, 0, size_t(std::max<int64_t>(c->n_total, 1)) * sizeof(int64_t), st)) !=
+            cudaSuccess)
+            return cuda_fail(c, e, "cudaMemsetAsync");
+    }
+    rc = run_launch(c, st, nullptr, c->n_inst, true);
+    if (rc) return rc;
+    c->h_res.resize(size_t(c->n_inst));
+    e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: copy of the results");
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: simulation kernel");
+    // instances whose active set outgrew the shared-memory workspace: re-run from global memory
+    std::vector<int32_t> redo;
+    for (int32_t i = 0; i < c->n_inst; ++i)
+        if (c->h_res[i].status == simgb::kStatusCapacity) redo.push_back(i);
+    if (!redo.empty()) {
+        e = cudaMemcpyAsync(c->d_work, redo.data(), redo.size() * sizeof(int32_t), cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: work list");
+        rc = run_launch(c, st, c->d_work, int32_t(redo.size()), false);
+        if (rc) return rc;
+        e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost,
+                            st);
+        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: copy of the results");
+        e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: simulation kernel (global workspace)");
+    }
+    int worst = SIM_OK;
+    for (int32_t i = 0; i < c->n_inst; ++i) {
+        const DevResult &d = c->h_res[i];
+        sim_result &r = out[i];
+        r.total_latency = d.total_latency;
+        r.makespan = d.makespan;
+        r.peak_memory = d.peak_memory;
+        r.evictions = d.evictions;
+        r.steps = d.steps;
+        r.request_steps = d.request_steps;
+        r.status = d.status;
+        r._pad = 0;
+        if (d.status == simgb::kStatusCapacity) r.status = SIM_E_STATE;
+        worst = std::min(worst, int(r.status));
+    }
+    c->ran = true;
+    c->comp_valid = c->record_completions != 0;
+    if (worst == SIM_E_STATE) fail(c, SIM_E_STATE, "sim_run: an internal consistency check failed");
+    else if (worst == SIM_E_STEPCAP) fail(c, SIM_E_STEPCAP, "sim_run: an instance hit the step cap");
+    else if (worst == SIM_E_INFEASIBLE) fail(c, SIM_E_INFEASIBLE, "sim_run: an instance has a request with s+o > M (or s+u > M under A_max)");
+    else if (worst == SIM_E_INVAL) fail(c, SIM_E_INVAL, "sim_run: an instance violates 1 <= l <= o <= u, s >= 1, a >= 0");
+    return worst;
+}
+
+int sim_get_completions(sim_ctx *c, int64_t *completion_t) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    if (!completion_t) return fail(c, SIM_E_INVAL, "sim_get_completions: NULL output");
+    if (!c->comp_valid || !c->d_comp)
+        return fail(c, SIM_E_STATE, "sim_get_completions: set SIM_OPT_RECORD_COMPLETIONS=1 and call sim_run first");
+    if (c->n_total == 0) return SIM_OK;
+    cudaError_t e =
+        cudaMemcpy(completion_t, c->d_comp, size_t(c->n_total) * sizeof(int64_t), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_get_completions: copy");
+    return SIM_OK;
+}
+
+int sim_competitive_ratio(const sim_ctx *cp, const sim_ctx *ch, double *cr_out, void *stream) {
+    sim_ctx *c = const_cast<sim_ctx *>(cp);
+    if (!cp || !ch || !cr_out) return SIM_E_INVAL;
+    c->err.clear();
+    if (cp->n_inst != ch->n_inst) return fail(c, SIM_E_INVAL, "sim_competitive_ratio: instance counts differ");
+    if (ch->policy != SIM_HSF) return fail(c, SIM_E_INVAL, "sim_competitive_ratio: reference context is not H-SF");
+    if (!cp->ran || !ch->ran) return fail(c, SIM_E_STATE, "sim_competitive_ratio: run both contexts first");
+    if (cp->device != ch->device) return fail(c, SIM_E_INVAL, "sim_competitive_ratio: contexts on different devices");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if (!c->d_cr && (e = dalloc(c->d_cr, size_t(c->n_inst) * sizeof(double))) != cudaSuccess)
+        return fail(c, SIM_E_NOMEM, "sim_competitive_ratio: buffer");
+    e = simgb::launch_ratio(cp->d_res, ch->d_res, c->d_cr, c->n_inst, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_competitive_ratio: launch");
+    ++c->launches;
+    e = cudaMemcpyAsync(cr_out, c->d_cr, size_t(c->n_inst) * sizeof(double), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_competitive_ratio: copy");
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_competitive_ratio: sync");
+    return SIM_OK;
+}
+
+int64_t sim_kernel_launches(const sim_ctx *c) { return c ? c->launches : -1; }
+
+const char *sim_last_error(const sim_ctx *c) { return c ? c->err.c_str() : g_create_err.c_str(); }
+
+void sim_destroy(sim_ctx *c) {
+    if (!c) return;
+    dfree(c->d_off);
+    dfree(c->d_raw);
+    dfree(c->d_rec);
+    dfree(c->d_rec_a);
+    dfree(c->d_info);
+    dfree(c->d_res);
+    dfree(c->d_comp);
+    dfree(c->d_counter);
+    dfree(c->d_work);
+    dfree(c->d_gws);
+    dfree(c->d_main);
+    dfree(c->d_cr);
+    delete c;
+}
+
+}  // extern "C"

@@ -1,0 +1,77 @@
+// Internal declarations shared by the C ABI (sim_api.cpp) and the CUDA kernels (sim_kernels.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace simgb {
+
+// Internal per-instance status: the active set outgrew the per-instance capacity of the launch;
+// the host re-runs such instances with a larger, global-memory workspace.
+constexpr int32_t kStatusCapacity = -100;
+constexpr int64_t kMaxM = int64_t(1) << 26;
+
+// One waiting request as the queue stores it; queues are ordered by (key, idx).
+struct QEnt {
+    int32_t key;  // length estimate used as the sort key: u (A_max), o (H-SF), current lower bound (A_min)
+    int32_t idx;  // request index within its instance
+    int32_t s;    // prompt size
+    int32_t o;    // true output length
+};
+
+// Per-instance constants produced by the staging kernel.
+struct InstInfo {
+    int64_t base;     // offset of the instance's first request
+    int64_t sum_a;    // sum of arrival steps (TEL = sum of completions - sum_a)
+    int64_t cap;      // step cap
+    int64_t work;     // cost estimate used to order instances (longest first)
+    int32_t n;        // number of requests
+    int32_t status;   // 0 or a sim_status from validation
+};
+
+struct DevResult {
+    int64_t total_latency, makespan, peak_memory, evictions, steps, request_steps;
+    int32_t status, pad;
+};
+
+struct StageParams {
+    int policy;
+    int64_t M;
+    int32_t n_inst;
+    int64_t step_cap;          // 0: default 64 * (n + sum o)
+    const int64_t *off;        // n_inst + 1
+    const int32_t *a, *s, *l, *u, *o;  // raw copies, n_total each
+    QEnt *rec;                 // out: per instance, sorted by (a, key, idx)
+    int32_t *rec_a;            // out: arrival step of rec[i]
+    InstInfo *info;            // out: n_inst
+};
+
+struct RunParams {
+    int64_t M;
+    int32_t n_work;            // instances to run in this launch
+    const int32_t *work;       // instance ids (n_work)
+    int32_t *counter;          // work-queue cursor (zeroed before launch)
+    const QEnt *rec;
+    const int32_t *rec_a;
+    const InstInfo *info;
+    DevResult *res;
+    int64_t *completion;       // optional, n_total
+    // workspace
+    int32_t ca;                // active-set capacity per instance (multiple of 32)
+    int32_t dcap;              // delta-queue capacity per instance (multiple of 32)
+    int32_t use_smem;          // 1: active set + delta queue in shared memory; 0: global workspace
+    unsigned char *gws;        // global workspace base (use_smem == 0)
+    int64_t gws_stride;        // bytes per warp slot
+    QEnt *mainbuf;             // ping-pong main-queue buffers, 2 * main_cap per warp slot
+    int64_t main_cap;
+};
+
+size_t warp_ws_bytes(int ca, int dcap);
+
+cudaError_t launch_stage(const StageParams &p, cudaStream_t st);
+cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
+                       cudaStream_t st);
+cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
+cudaError_t set_run_smem_limit(int policy, size_t bytes);
+
+}  // namespace simgb

@@ -1,0 +1,84 @@
+"""A small object wrapper over the C ABI: one ``Simulator`` per (policy, M, n_instances) context."""
+from __future__ import annotations
+
+import numpy as np
+
+from . import _lib as L
+
+
+def _i32_host(x) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+
+
+class Simulator:
+    """Owns a sim_ctx.  ``load`` accepts numpy arrays (host) or int32 CUDA tensors (device)."""
+
+    def __init__(self, policy: int, M: int, n_instances: int, **options):
+        self.policy, self.M, self.n_instances = int(policy), int(M), int(n_instances)
+        self.ctx = L.sim_create(policy, M, n_instances)
+        self._keep = None
+        for k, v in options.items():
+            self.set_option(k, v)
+
+    OPTIONS = {"step_cap": L.SIM_OPT_STEP_CAP, "record_completions": L.SIM_OPT_RECORD_COMPLETIONS,
+               "warps_per_block": L.SIM_OPT_WARPS_PER_BLOCK, "smem_active_cap": L.SIM_OPT_SMEM_ACTIVE_CAP}
+
+    def set_option(self, name: str, value: int) -> None:
+        rc = L.sim_set_option(self.ctx, self.OPTIONS[name], int(value))
+        if rc != L.SIM_OK:
+            raise L.SimError(rc, L.sim_last_error(self.ctx))
+
+    def _check(self, rc: int, allow_instance_status: bool = False) -> int:
+        if rc != L.SIM_OK and not (allow_instance_status and rc in (L.SIM_E_INVAL, L.SIM_E_INFEASIBLE,
+                                                                     L.SIM_E_STEPCAP)):
+            raise L.SimError(rc, L.sim_last_error(self.ctx))
+        return rc
+
+    def load(self, offsets, a, s, l, u, o) -> None:
+        offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+        dev = hasattr(a, "is_cuda") and a.is_cuda
+        if dev:
+            arrs = [x.contiguous() for x in (a, s, l, u, o)]
+            for x in arrs:
+                assert str(x.dtype) == "torch.int32"
+        else:
+            arrs = [_i32_host(x) for x in (a, s, l, u, o)]
+        self._check(L.sim_load_csr(self.ctx, offsets, *arrs, 1 if dev else 0))
+
+    def load_workload(self, w) -> None:
+        self.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o)
+
+    def run(self, stream: int = 0) -> np.ndarray:
+        out = np.zeros(self.n_instances, dtype=L.RESULT_DTYPE)
+        self.last_rc = self._check(L.sim_run(self.ctx, out, stream), allow_instance_status=True)
+        return out
+
+    def completions(self, n_total: int) -> np.ndarray:
+        out = np.zeros(max(n_total, 1), dtype=np.int64)
+        self._check(L.sim_get_completions(self.ctx, out))
+        return out[:n_total]
+
+    def competitive_ratio(self, hsf: "Simulator", stream: int = 0) -> np.ndarray:
+        out = np.zeros(self.n_instances, dtype=np.float64)
+        self._check(L.sim_competitive_ratio(self.ctx, hsf.ctx, out, stream))
+        return out
+
+    def kernel_launches(self) -> int:
+        return L.sim_kernel_launches(self.ctx)
+
+    def close(self) -> None:
+        if getattr(self, "ctx", None):
+            L.sim_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

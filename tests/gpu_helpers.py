@@ -1,0 +1,42 @@
+"""Helpers for the GPU parity tests: run a Workload through the C ABI and through the C oracle."""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+
+FIELDS = ("total_latency", "makespan", "peak_memory", "evictions", "steps", "request_steps", "status")
+
+
+def n_threads() -> int:
+    return max(1, min(32, os.cpu_count() or 1))
+
+
+def gpu_run(policy, w, device_load=True, completions=False, **opts):
+    import torch
+
+    from paper_2508_14544_gb300 import Simulator
+    with Simulator(policy, w.M, w.n_instances, record_completions=int(completions), **opts) as sim:
+        if device_load:
+            dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in
+                   (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
+            sim.load(w.offsets, *dev)
+        else:
+            sim.load_workload(w)
+        res = sim.run()
+        comp = sim.completions(w.n_total) if completions else None
+    return res, comp
+
+
+def oracle_run(policy, w, completions=False, step_cap=0):
+    from oracle import plain
+    return plain.run_workload(policy, w, step_cap=step_cap, n_threads=n_threads(), completions=completions)
+
+
+def assert_same(got, ref, rows=None, tag=""):
+    rows = np.arange(len(ref)) if rows is None else np.asarray(rows)
+    for f in FIELDS:
+        g = np.asarray(got[f])[rows] if len(got) != len(ref) else np.asarray(got[f])
+        r = np.asarray(ref[f])
+        bad = np.nonzero(g != r)[0]
+        assert bad.size == 0, f"{tag}: field {f} differs at rows {bad[:10].tolist()}: gpu {g[bad[:5]].tolist()} oracle {r[bad[:5]].tolist()}"

@@ -1,0 +1,153 @@
+"""C-ABI behaviour on the GPU: statuses, options, host vs device loads, reruns, edge cases."""
+import numpy as np
+import pytest
+
+from tests.gpu_helpers import FIELDS, assert_same, gpu_run, oracle_run
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+
+
+def _w(parts, M):
+    from paper_2508_14544_gb300 import workloads as W
+    return W.concat_instances("edge", M, parts)
+
+
+def test_empty_and_ragged_instances():
+    parts = [dict(a=[], s=[], l=[], u=[], o=[]),
+             dict(a=[0], s=[3], l=[2], u=[5], o=[4]),
+             dict(a=[], s=[], l=[], u=[], o=[]),
+             dict(a=[5, 5, 9], s=[1, 2, 3], l=[1, 1, 1], u=[3, 3, 3], o=[2, 3, 1])]
+    w = _w(parts, 12)
+    for pol in (0, 1, 2):
+        got, comp = gpu_run(pol, w, completions=True)
+        ref, rcomp = oracle_run(pol, w, completions=True)
+        assert_same(got, ref, tag="edge")
+        assert np.array_equal(comp, rcomp)
+        assert got["steps"][0] == 0 and got["status"][0] == 0
+
+
+def test_per_instance_validation_statuses():
+    parts = [dict(a=[0], s=[1], l=[2], u=[3], o=[1]),      # l > o   -> INVAL
+             dict(a=[0], s=[1], l=[1], u=[1], o=[2]),      # o > u   -> INVAL
+             dict(a=[-1], s=[1], l=[1], u=[1], o=[1]),     # a < 0   -> INVAL
+             dict(a=[0], s=[0], l=[1], u=[1], o=[1]),      # s < 1   -> INVAL
+             dict(a=[0], s=[5], l=[1], u=[9], o=[6]),      # s+o > M -> INFEASIBLE
+             dict(a=[0], s=[5], l=[1], u=[9], o=[4]),      # s+u > M: A_max only
+             dict(a=[0, 1], s=[1, 1], l=[1, 1], u=[2, 2], o=[1, 2])]
+    w = _w(parts, 10)
+    for pol in (0, 1, 2):
+        got, _ = gpu_run(pol, w)
+        ref = oracle_run(pol, w)
+        assert_same(got, ref, tag=f"validation pol={pol}")
+        assert list(got["status"][:5]) == [-1, -1, -1, -1, -2]
+        assert got["status"][5] == (-2 if pol == 0 else 0)
+
+
+def test_step_cap_matches_oracle():
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", [0, 300, 600, 900])
+    for cap in (1, 3, 500):
+        for pol in (0, 1, 2):
+            got, _ = gpu_run(pol, w, step_cap=cap)
+            ref = oracle_run(pol, w, step_cap=cap)
+            assert_same(got, ref, tag=f"cap={cap}")
+            assert np.all(got["status"] == -3)
+            assert np.all(got["steps"] == cap)
+
+
+def test_capacity_fallback_identical():
+    """A 32-slot shared-memory active set forces most instances onto the global-memory path."""
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(0, 1024, 32))
+    for pol in (0, 1, 2):
+        a, ca = gpu_run(pol, w, completions=True)
+        b, cb = gpu_run(pol, w, completions=True, smem_active_cap=32)
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f])
+        assert np.array_equal(ca, cb)
+
+
+def test_host_and_device_loads_and_reruns_agree():
+    from paper_2508_14544_gb300 import Simulator
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(0, 1024, 64))
+    for pol in (0, 1, 2):
+        a, _ = gpu_run(pol, w, device_load=True)
+        b, _ = gpu_run(pol, w, device_load=False)
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f])
+        with Simulator(pol, w.M, w.n_instances) as sim:
+            sim.load_workload(w)
+            r1 = sim.run()
+            r2 = sim.run()
+        for f in FIELDS:
+            assert np.array_equal(r1[f], r2[f]) and np.array_equal(r1[f], a[f])
+
+
+@pytest.mark.parametrize("wpb", [1, 2, 8])
+def test_launch_shapes_agree(wpb):
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(5, 1024, 41))
+    for pol in (0, 1, 2):
+        a, _ = gpu_run(pol, w)
+        b, _ = gpu_run(pol, w, warps_per_block=wpb)
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f])
+
+
+def test_sparse_arrivals_and_bursts():
+    """Idle gaps (time jumps), one large burst (bulk insert through the delta queue), and many
+    evictions for A_min, at sizes that exercise delta merges."""
+    from fractions import Fraction
+
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(3)
+    parts = []
+    for i in range(24):
+        n = 1500
+        s = rng.integers(1, 40, n)
+        o = rng.integers(1, 200, n)
+        l, u = W.interval_for(o, Fraction(1, 4), rng)
+        a = np.sort(rng.integers(0, 4000, n))
+        if i % 3 == 0:
+            a[300:900] = a[300]  # a burst of 600 arrivals in one step
+        if i % 3 == 1:
+            a = a * 7  # long idle gaps
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    w = W.concat_instances("arrivals", 3000, parts)
+    for pol in (0, 1, 2):
+        got, comp = gpu_run(pol, w, completions=True)
+        ref, rcomp = oracle_run(pol, w, completions=True)
+        assert_same(got, ref, tag=f"arrivals pol={pol}")
+        assert np.array_equal(comp, rcomp)
+
+
+def test_unsorted_arrivals():
+    """Arrival steps not in index order: staging sorts by (arrival, key, index)."""
+    from fractions import Fraction
+
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(4)
+    parts = []
+    for i in range(40):
+        n = int(rng.integers(1, 300))
+        s = rng.integers(1, 20, n)
+        o = rng.integers(1, 60, n)
+        l, u = W.interval_for(o, Fraction(1, 2), rng)
+        a = rng.integers(0, 200, n)
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    w = W.concat_instances("unsorted", 600, parts)
+    for pol in (0, 1, 2):
+        got, comp = gpu_run(pol, w, completions=True)
+        ref, rcomp = oracle_run(pol, w, completions=True)
+        assert_same(got, ref, tag="unsorted")
+        assert np.array_equal(comp, rcomp)

@@ -1,0 +1,147 @@
+"""CUDA path (through the C ABI) vs the CPU oracle: bit-exact on every integer output."""
+import numpy as np
+import pytest
+
+from tests import pins
+from tests.gpu_helpers import FIELDS, assert_same, gpu_run, oracle_run
+
+pytestmark = pytest.mark.gpu
+
+POLS = (0, 1, 2)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+
+
+def _gpu_sim(p, M, a, s, l, u, o):
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.concat_instances("pin", M, [dict(a=a, s=s, l=l, u=u, o=o)])
+    res, comp = gpu_run(p, w, completions=True)
+    out = {k: int(res[0][k]) for k in FIELDS}
+    out["completion"] = comp.tolist()
+    return out
+
+
+def test_paper_pins_on_gpu():
+    """Example 1, the Definition-1 example, the hand traces and the wave closed forms."""
+    fails = pins.check_all(_gpu_sim)
+    assert not fails, fails
+
+
+def _random_tiny_workload(seed, n_inst=1500, arrivals=True):
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(seed)
+    parts = []
+    M = 40
+    for i in range(n_inst):
+        n = int(rng.integers(0, 12))
+        o = rng.integers(1, 10, n)
+        l = np.array([rng.integers(1, x + 1) for x in o], dtype=np.int64)
+        u = o + rng.integers(0, 8, n)
+        s = rng.integers(1, 6, n)
+        u = np.minimum(u, M - s)
+        a = rng.integers(0, 12, n) if arrivals else np.zeros(n, int)
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    return W.concat_instances("tiny", M, parts)
+
+
+@pytest.mark.parametrize("arrivals", [False, True])
+@pytest.mark.parametrize("pol", POLS)
+def test_random_tiny_batch(pol, arrivals):
+    w = _random_tiny_workload(100 + arrivals, arrivals=arrivals)
+    got, comp = gpu_run(pol, w, completions=True)
+    ref, rcomp = oracle_run(pol, w, completions=True)
+    assert_same(got, ref, tag=f"tiny pol={pol}")
+    assert np.array_equal(comp, rcomp)
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_c1(pol):
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c1")
+    got, comp = gpu_run(pol, w, completions=True)
+    ref, rcomp = oracle_run(pol, w, completions=True)
+    assert_same(got, ref, tag="c1")
+    assert np.array_equal(comp, rcomp)
+
+
+@pytest.fixture(scope="module")
+def c2():
+    from paper_2508_14544_gb300 import workloads as W
+    return W.make_workload("c2")
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_c2_full(c2, pol):
+    """All 1024 instances of the 1000-request workload, in the launch configuration the bench uses."""
+    got, _ = gpu_run(pol, c2)
+    ref = oracle_run(pol, c2)
+    assert_same(got, ref, tag=f"c2 pol={pol}")
+
+
+def test_c2_competitive_ratio(c2):
+    from paper_2508_14544_gb300 import Simulator
+    sims = {}
+    for pol in POLS:
+        s = Simulator(pol, c2.M, c2.n_instances)
+        s.load_workload(c2)
+        s.run()
+        sims[pol] = s
+    ref = {pol: oracle_run(pol, c2) for pol in POLS}
+    for pol in (0, 1):
+        cr = sims[pol].competitive_ratio(sims[2])
+        want = ref[pol]["total_latency"].astype(np.float64) / ref[2]["total_latency"].astype(np.float64)
+        assert np.array_equal(cr, want)  # same IEEE division of the same integers
+        assert np.all(cr >= 1.0 - 1e-12) or pol == 1
+    for s in sims.values():
+        s.close()
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_c3_full(pol):
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c3")
+    got, _ = gpu_run(pol, w)
+    ref = oracle_run(pol, w)
+    assert_same(got, ref, tag=f"c3 pol={pol}")
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_c4_full_sampled(pol):
+    """All 40960 instances on the GPU; every 160th instance (256 of them, all alphas) against the
+    oracle, plus invariants on all."""
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c4")
+    got, _ = gpu_run(pol, w)
+    rows = np.arange(0, w.n_instances, 160)
+    ref = oracle_run(pol, w.subset(rows))
+    for f in FIELDS:
+        assert np.array_equal(got[f][rows], ref[f]), f
+    assert np.all(got["status"] == 0)
+    assert np.all(got["peak_memory"] <= w.M)
+    so = np.add.reduceat(w.true_o.astype(np.int64), w.offsets[:-1])
+    if pol in (0, 2):
+        assert np.all(got["evictions"] == 0)
+        assert np.array_equal(got["request_steps"], so)
+    else:
+        assert np.all(got["request_steps"] >= so)
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_c5_full_sampled(pol):
+    """All 64 instances of the 10^5-request online workload on the GPU; two against the oracle."""
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c5")
+    got, _ = gpu_run(pol, w)
+    rows = [0, 37]
+    ref = oracle_run(pol, w.subset(rows))
+    for f in FIELDS:
+        assert np.array_equal(got[f][rows], ref[f]), f
+    assert np.all(got["status"] == 0)
+    assert np.all(got["peak_memory"] <= w.M)
