@@ -1,0 +1,51 @@
+"""Command-line runner: simulate a named synthetic workload under one policy through the C ABI.
+
+  python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024] [--repeat 1]
+
+Prints one JSON line per run with the wall time of sim_run and totals of the result fields.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import time
+
+import numpy as np
+
+from . import POLICIES, Simulator
+from . import workloads as W
+
+
+def main(argv=None) -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", default="c2", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--policy", default="A_min", choices=sorted(POLICIES))
+    ap.add_argument("--instances", default=None, help="a:b range of instance ids (default: all)")
+    ap.add_argument("--repeat", type=int, default=1)
+    ap.add_argument("--warps-per-block", type=int, default=0)
+    args = ap.parse_args(argv)
+    ids = None
+    if args.instances:
+        a, b = (int(x) for x in args.instances.split(":"))
+        ids = range(a, b)
+    w = W.make_workload(args.workload, ids)
+    import torch
+    dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
+    opts = {}
+    if args.warps_per_block:
+        opts["warps_per_block"] = args.warps_per_block
+    with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
+        for _ in range(args.repeat):
+            sim.load(w.offsets, *dev)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            res = sim.run()
+            dt = time.perf_counter() - t0
+            print(json.dumps({"workload": args.workload, "policy": args.policy, "instances": w.n_instances,
+                              "sim_run_s": dt, "request_steps": int(res["request_steps"].sum()),
+                              "steps": int(res["steps"].sum()), "evictions": int(res["evictions"].sum()),
+                              "worst_status": int(res["status"].min())}), flush=True)
+
+
+if __name__ == "__main__":
+    main()
