@@ -31,6 +31,7 @@ __all__ = [
     "WORKLOADS",
     "make_workload",
     "make_instance",
+    "rank_instances",
     "interval_for",
     "concat_instances",
 ]
@@ -176,6 +177,13 @@ WORKLOADS: dict[str, _Spec] = {
                 "64 instances x n=10^5, Poisson arrivals rate 2/step, M=500000, s~U{1..2048}, "
                 "o~Zipf(1.2) in [1,8192], alpha=3/10"),
 }
+
+
+def rank_instances(name: str, rank: int) -> range:
+    """Instance ids simulated by one rank when every GPU runs its own copy of a workload's shape
+    (weak scaling): rank r takes ids [r*N, (r+1)*N) of the workload's seed sequence."""
+    n = WORKLOADS[name].n_instances
+    return range(rank * n, (rank + 1) * n)
 
 
 def make_instance(name: str, i: int) -> dict:
