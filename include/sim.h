@@ -146,6 +146,32 @@ int sim_competitive_ratio(const sim_ctx *ctx_policy, const sim_ctx *ctx_hsf, dou
  * (staging, simulation, fallback and ratio kernels).  ctx NULL -> -1. */
 int64_t sim_kernel_launches(const sim_ctx *ctx);
 
+/*
+ * sim_run_noalloc: stage and simulate in one call WITHOUT allocating any device memory.  The
+ * paper has no counterpart: this is a library convenience for callers that cannot call cudaMalloc
+ * -- a process whose GPU memory is all reserved up front by its own pool allocator (a cudaMalloc
+ * would fail or fragment that reservation), or a latency-sensitive loop that must avoid the
+ * implicitly synchronising allocation calls (cudaFree waits for the whole device).
+ * Semantics and results are those of sim_load_csr + sim_run with default options.
+ *   policy, M, n_instances  as for sim_create (1 <= n_instances <= 16384).
+ *   offsets     HOST, n_instances + 1 int64, as for sim_load_csr.
+ *   arrival_t .. true_o     DEVICE int32 arrays (current device), layout as for sim_load_csr.
+ *   results     DEVICE, n_instances sim_result, written by the kernels.
+ *   cuda_stream a cudaStream_t or NULL.  The call only enqueues work: read `results` after
+ *               synchronising the stream.  Per-instance statuses are in results[i].status.
+ * Everything except the inputs and outputs lives in one fixed array of about 23 MB that every GPU
+ * loading the library holds until the process exits.  Limits: at most 2048 requests per instance
+ * and 262,144 requests per call; larger inputs are rejected with SIM_E_INVAL and a message in
+ * sim_last_error(NULL).  All calls share that array and it keeps the last call's contents: calls
+ * that overlap on the GPU (different streams or threads) race; calls on one stream are safe.
+ * The first call on each device looks up the array's device address (cudaGetSymbolAddress) with
+ * that device current; make that first call before any stream capture.  Allocates nothing.
+ * Returns SIM_OK, SIM_E_INVAL, SIM_E_CUDA or SIM_E_STATE.
+ */
+int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const int64_t *offsets, const int32_t *arrival_t,
+                    const int32_t *prompt_s, const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o,
+                    sim_result *results, void *cuda_stream);
+
 /* sim_set_option: set one of the SIM_OPT_* options.  Returns SIM_OK or SIM_E_INVAL. */
 int sim_set_option(sim_ctx *ctx, int key, int64_t value);
 

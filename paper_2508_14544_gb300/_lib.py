@@ -34,7 +34,7 @@ RESULT_DTYPE = np.dtype([
 assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
 
 EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
-           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches")
+           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc")
 
 _lib = None
 
@@ -80,6 +80,8 @@ def lib() -> ctypes.CDLL:
     L.sim_destroy.restype = None
     L.sim_kernel_launches.argtypes = [vp]
     L.sim_kernel_launches.restype = ctypes.c_int64
+    L.sim_run_noalloc.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, vp, vp, vp, vp, vp, vp, vp, vp]
+    L.sim_run_noalloc.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -139,6 +141,15 @@ def sim_competitive_ratio(ctx_policy, ctx_hsf, out: np.ndarray, stream: int = 0)
 
 def sim_kernel_launches(ctx) -> int:
     return int(lib().sim_kernel_launches(ctx))
+
+
+def sim_run_noalloc(policy: int, M: int, offsets: np.ndarray, a, s, l, u, o, results, stream: int = 0) -> int:
+    """Stage and simulate without any device allocation by the library (see include/sim.h).
+    a..o and results are device tensors; offsets is a host int64 array."""
+    assert offsets.dtype == np.int64 and offsets.flags.c_contiguous
+    n_inst = int(offsets.shape[0] - 1)
+    return lib().sim_run_noalloc(int(policy), int(M), n_inst, offsets.ctypes.data, _ptr(a), _ptr(s), _ptr(l),
+                                 _ptr(u), _ptr(o), _ptr(results), ctypes.c_void_p(stream or None))
 
 
 def sim_destroy(ctx) -> None:

@@ -108,6 +108,11 @@ int check_device(sim_ctx *c) {
 
 }  // namespace
 
+namespace simgb {
+// Message for sim_last_error(NULL) from entry points that have no context.
+void set_global_error(const char *msg) { g_create_err = msg ? msg : ""; }
+}  // namespace simgb
+
 extern "C" {
 
 int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out) {
