@@ -149,8 +149,8 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
             c->wpb = int(value);
             return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
-            if (value < 32 || value > 4096 || value % 32)
-                return fail(c, SIM_E_INVAL, "SMEM_ACTIVE_CAP must be a multiple of 32 in [32, 4096]");
+            if (value < 128 || value > 4096 || value % 128)
+                return fail(c, SIM_E_INVAL, "SMEM_ACTIVE_CAP must be a multiple of 128 in [128, 4096]");
             c->smem_ca = int(value);
             return SIM_OK;
         default:
@@ -251,7 +251,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     int wpb = c->wpb;
     const int dcap = c->dcap;
-    int ca = smem ? c->smem_ca : ((std::max(c->n_max, 32) + 31) / 32) * 32;
+    int ca = smem ? c->smem_ca : ((std::max(c->n_max, 128) + 127) / 128) * 128;
     size_t per_warp = simgb::warp_ws_bytes(ca, dcap);
     size_t smem_bytes = 0;
     if (smem) {

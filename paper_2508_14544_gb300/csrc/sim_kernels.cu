@@ -1,30 +1,35 @@
-// CUDA kernels of the batched scheduler simulator (sm_103a).
+// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy>.
 //
-//   k_stage  - per instance: validate the requests (Section 2 model), compute TEL/step-cap
-//              constants, and sort the requests by (arrival step, policy key, index) so that every
-//              arrival batch is already ordered the way the waiting set R_t is sorted
-//              (Algorithm malb: key u; Algorithm milb/milbrevise: key l; Algorithm off: key o).
-//   k_run    - one warp simulates one instance at a time, step by step (persistent warps pulling
-//              instance ids from a work queue).  Per step: arrivals join R_t; A_min resolves an
-//              overflow of the next step by cancelling in ascending (estimate, index) order
-//              (Algorithm milb); the head of R_t is admitted while the future-memory check of
-//              eq. Constraint holds (largest feasible prefix); the batch is processed (one token per
-//              member, eq. constraintM accounting, completions, TEL of eq. latency).
-//   k_ratio  - per-instance competitive ratio TEL(pi) / TEL(H-SF) (Definition cr).
+// One warp simulates one instance at a time (persistent warps pull instance ids from a work
+// queue).  Each step follows the paper's algorithms:
+//   S1  arrivals with a_i <= t join the waiting set R_t (extension: the paper has a_i = 0);
+//   S3  A_min only (Algorithm milb): if the next step of the active set would exceed M, cancel
+//       jobs in ascending (estimate, index) order until it fits; each cancelled job's estimate
+//       becomes max(estimate, tokens generated) and it re-enters R_t in the same step;
+//   S5  admit the head of R_t (sorted by (key, index)) while eq. Constraint holds at every future
+//       step: the largest feasible prefix (Algorithms malb / milb / off);
+//   S6  process the batch: one token per member, the step's memory sum(s + tokens) (eq.
+//       constraintM), completions, TEL (eq. latency).
 //
-// Active set layout (per warp, shared memory when it fits): structure-of-arrays sorted by the
-// projected last step E (ascending):
+// Active set (per warp, shared memory; a global-memory workspace of the same layout serves
+// instances that outgrow it), structure of arrays sorted by the projected last step E:
 //   E = p + Lhat - 1   projected last step (Lhat = u, o or the A_min estimate)
-//   F = p + o - 1      true last step (completion at step F, C = F + 1)
-//   B = s - p + 1      so the job's memory at step x is B + x
-//   P = p, I = request index, K = the estimate (A_min sort key)
-// Derived arrays, rebuilt whenever the set changes, relative to a time base tb:
-//   SB[i] = sum_{j >= i} (B_j + tb)                      (suffix sums; SB[A] = 0)
-//   PM[h] = max_{i < h} (SB[i] + (A - i)(E_i - tb) + E_i - tb)   (prefix maxima; PM[0] = -inf)
-// With these, the future memory of the active set at its endpoint E_i is
-// V(E_i) = SB[i] + (A - i)(E_i - tb) (exact for the first entry of each group of equal E, and a
-// lower bound for the others, so maxima are exact), and the check "the head of R_t, started now,
-// keeps every future step within M" costs O(1) per step (see head_fits).
+//   F = p + o - 1      true last step (completion at step F, C = F + 1); F < 0 marks a removed job
+//   B = s - p + 1      the job's memory at step x is B + x
+//   P = p, I = request index, K = the estimate (A_min key)
+// Derived arrays, recomputed in one warp pass whenever the set changes, relative to a time base tb:
+//   SB[i] = sum_{j >= i} (B_j + tb),  SB[A] = 0                    (suffix sums)
+//   PM[h] = max_{i < h} H_i,  H_i = SB[i] + (A - i)(E_i - tb) + (E_i - tb),  PM[0] = -inf
+// V(x) = SB[lb] + (A - lb)(x - tb), lb = #{E < x}, is the projected memory of the active set at
+// step x (eq. Constraint restricted to S'); H_i is V(E_i) + E_i - tb for the first entry of each
+// group of equal E and a lower bound for the others, so prefix maxima are exact.  The head
+// candidate (prompt s, estimate L) started at step t fits iff
+//   (1) SB[0] + A (t - tb) + s + 1 <= M                 (the coming step),
+//   (2) PM[#{E <= y}] + s + 1 - (t - tb) <= M            (every active endpoint it covers),
+//   (3) V(y) + s + L <= M,  y = t + L - 1                (its own last step),
+// so a step in which nothing changes costs O(1), and a run of such steps is processed in closed
+// form up to the next event (completion, arrival, A_min overflow, or the first step at which
+// the head fits, found by scanning the segments between active endpoints).
 #include <climits>
 #include <cstdint>
 
@@ -36,31 +41,25 @@ namespace {
 
 constexpr unsigned FULL = 0xffffffffu;
 enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
-enum { ST_OK = 0, ST_INVAL = -1, ST_INFEASIBLE = -2, ST_STEPCAP = -3, ST_STATE = -5 };
+enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
+constexpr int kChunk = 128;  // active-set entries per warp pass (4 per lane)
+constexpr int64_t kBig = int64_t(1) << 60;
+
+__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 
 __device__ __forceinline__ bool qless(const QEnt &a, const QEnt &b) {
     return a.key < b.key || (a.key == b.key && a.idx < b.idx);
 }
 
-__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
-
-__device__ __forceinline__ int64_t warp_sum64(int64_t v) {
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) v += __shfl_xor_sync(FULL, v, d);
-    return v;
-}
-
-__device__ __forceinline__ int warp_min32(int v) {
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) v = min(v, __shfl_xor_sync(FULL, v, d));
-    return v;
-}
-
 __device__ __forceinline__ int sat32(int64_t v) {
     const int64_t hi = int64_t(1) << 30;
-    if (v > hi) return int(hi);
-    if (v < -hi) return int(-hi);
-    return int(v);
+    return int(v > hi ? hi : (v < -hi ? -hi : v));
+}
+
+__device__ __forceinline__ int64_t floor_div(int64_t a, int64_t b) {  // b > 0
+    int64_t q = a / b;
+    if ((a % b != 0) && (a < 0)) --q;
+    return q;
 }
 
 __device__ __forceinline__ QEnt shfl_q(const QEnt &q, int src) {
@@ -72,8 +71,46 @@ __device__ __forceinline__ QEnt shfl_q(const QEnt &q, int src) {
     return r;
 }
 
-// Number of leading positions i in [0, len) with pred(i) true, for a predicate that is true on a
-// prefix.  Two ballots over 32 samples: O(1) dependent loads for len <= 1024.
+// Exclusive prefix sum over lanes; total = sum over all lanes.
+__device__ __forceinline__ int excl_scan_add(int v, int &total) {
+    const int lane = lane_id();
+    int x = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_up_sync(FULL, x, d);
+        if (lane >= d) x += y;
+    }
+    total = __shfl_sync(FULL, x, 31);
+    return x - v;
+}
+
+// Sum over lanes above this one; total = sum over all lanes.
+__device__ __forceinline__ int excl_suffix_add(int v, int &total) {
+    const int lane = lane_id();
+    int x = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_down_sync(FULL, x, d);
+        if (lane + d < 32) x += y;
+    }
+    total = __shfl_sync(FULL, x, 0);
+    return x - v;
+}
+
+// Max over lanes below this one (INT_MIN for lane 0).
+__device__ __forceinline__ int excl_scan_max(int v) {
+    const int lane = lane_id();
+    int x = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_up_sync(FULL, x, d);
+        if (lane >= d) x = max(x, y);
+    }
+    const int ex = __shfl_up_sync(FULL, x, 1);
+    return lane == 0 ? INT_MIN : ex;
+}
+
+// Number of leading positions i in [0, len) with pred(i) true (pred true on a prefix).
 template <class Pred>
 __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
     if (len <= 0) return 0;
@@ -98,23 +135,19 @@ __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
 // Per-warp workspace
 // ---------------------------------------------------------------------------------------------
 struct Ws {
-    int32_t *E, *F, *B, *P, *I, *K;  // active set, capacity ca
-    int32_t *SB, *PM;                // ca + 1
-    QEnt *dq;                        // delta queue, capacity dcap, sorted DESCENDING (head at the end)
-    int32_t *cnt;                    // dcap + 1 (merge histogram)
+    int32_t *E, *F, *B, *P, *I, *K;  // active set, capacity ca (multiple of kChunk), 16-byte aligned
+    int32_t *SB, *PM;                // ca + 4
+    QEnt *dq;                        // delta queue, dcap entries (power of two), unsorted
+    int32_t *cnt;                    // dcap + 4 (merge histogram)
     QEnt *mb0, *mb1;                 // global ping-pong main-queue buffers
     int32_t ca, dcap;
 };
 
 __host__ __device__ inline size_t ws_bytes_impl(int ca, int dcap) {
-    size_t b = 0;
-    b += size_t(6) * ca * sizeof(int32_t);
-    b += size_t(2) * (ca + 1) * sizeof(int32_t);
+    size_t b = size_t(6) * ca * sizeof(int32_t) + size_t(2) * (ca + 4) * sizeof(int32_t);
     b = (b + 15) & ~size_t(15);
-    b += size_t(dcap) * sizeof(QEnt);
-    b += size_t(dcap + 1) * sizeof(int32_t);
-    b = (b + 15) & ~size_t(15);
-    return b;
+    b += size_t(dcap) * sizeof(QEnt) + size_t(dcap + 4) * sizeof(int32_t);
+    return (b + 15) & ~size_t(15);
 }
 
 __device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
@@ -126,9 +159,9 @@ __device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
     w.P = p; p += ca;
     w.I = p; p += ca;
     w.K = p; p += ca;
-    w.SB = p; p += ca + 1;
-    w.PM = p; p += ca + 1;
-    size_t off = (reinterpret_cast<unsigned char *>(p) - base);
+    w.SB = p; p += ca + 4;
+    w.PM = p; p += ca + 4;
+    size_t off = size_t(reinterpret_cast<unsigned char *>(p) - base);
     off = (off + 15) & ~size_t(15);
     w.dq = reinterpret_cast<QEnt *>(base + off);
     w.cnt = reinterpret_cast<int32_t *>(w.dq + dcap);
@@ -137,47 +170,99 @@ __device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
     return w;
 }
 
+__device__ __forceinline__ int4 ld4(const int32_t *a, int i) { return *reinterpret_cast<const int4 *>(a + i); }
+
 // ---------------------------------------------------------------------------------------------
-// Waiting set R_t: a sorted main array in global memory [mh, me) plus a small sorted delta array
-// (the workspace, descending so that its head is the last element).  Together they hold R_t in
-// (key, idx) order.  Inserts go to the delta; a full delta is merged into the main array.
+// Waiting set R_t: a sorted main array in global memory [mh, me) (lane-cached head) plus an
+// unsorted delta array in the workspace with its minimum cached.  A full delta is sorted (warp
+// bitonic sort) and merged into the main array.  Order: (key, idx).
 // ---------------------------------------------------------------------------------------------
 struct Queue {
     const QEnt *mq;  // main array (global, ascending); may point into the staged records
     int mh, me;      // head / end
     int mbuf;        // -1: mq is read-only staged data; 0/1: ping-pong buffer in use
     int dn;          // delta size
+    int dminpos;     // position of the delta minimum
+    QEnt dmin;       // delta minimum
     int mcb;         // main head cache base (lane l caches mq[mcb + l]), -1 invalid
     QEnt mc;         // this lane's cached main entry
 };
 
 __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.me && q.dn == 0; }
 
+__device__ void delta_recompute_min(const Ws &w, Queue &q) {
+    const int lane = lane_id();
+    unsigned bk = UINT_MAX, bi = UINT_MAX;
+    int bp = -1;
+    for (int j = lane; j < q.dn; j += 32) {
+        const QEnt e = w.dq[j];
+        const unsigned k = unsigned(e.key), i = unsigned(e.idx);
+        if (k < bk || (k == bk && i < bi)) {
+            bk = k;
+            bi = i;
+            bp = j;
+        }
+    }
+    const unsigned mk = __reduce_min_sync(FULL, bk);
+    const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
+    const unsigned ball = __ballot_sync(FULL, bp >= 0 && bk == mk && bi == mi);
+    const int src = ball ? __ffs(ball) - 1 : 0;
+    q.dminpos = __shfl_sync(FULL, bp, src);
+    if (q.dn > 0) q.dmin = w.dq[q.dminpos];
+}
+
+// Sort the delta ascending in place (bitonic network over dcap entries, padded with +inf).
+__device__ void delta_sort(const Ws &w, int dn) {
+    const int lane = lane_id();
+    const int D = w.dcap;
+    QEnt inf;
+    inf.key = INT_MAX;
+    inf.idx = INT_MAX;
+    inf.s = 0;
+    inf.o = 0;
+    for (int j = dn + lane; j < D; j += 32) w.dq[j] = inf;
+    __syncwarp();
+    for (int k = 2; k <= D; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int p = lane; p < (D >> 1); p += 32) {
+                const int i = (p / j) * 2 * j + (p % j);
+                const int l = i + j;
+                const QEnt a = w.dq[i], b = w.dq[l];
+                const bool asc = (i & k) == 0;
+                if (qless(b, a) == asc) {
+                    w.dq[i] = b;
+                    w.dq[l] = a;
+                }
+            }
+            __syncwarp();
+        }
+    }
+}
+
 // Merge the delta into the main array (into the other ping-pong buffer).
 __device__ void merge_delta(const Ws &w, Queue &q) {
     const int lane = lane_id();
     const int dn = q.dn;
+    delta_sort(w, dn);
     const int nx = q.me - q.mh;
     QEnt *out = (q.mbuf == 0) ? w.mb1 : w.mb0;
     const QEnt *X = q.mq + q.mh;
-    // delta ascending view: Yasc(j) = dq[dn - 1 - j]
     for (int j = lane; j <= dn; j += 32) w.cnt[j] = 0;
     __syncwarp();
     const int c = (nx + 31) >> 5;
     const int s0 = lane * c;
     const int s1 = min(s0 + c, nx);
     if (s0 < s1) {
-        // r = #Y < X[s0]  (binary search over the ascending view)
         const QEnt x0 = X[s0];
         int lo = 0, hi = dn;
         while (lo < hi) {
             const int mid = (lo + hi) >> 1;
-            if (qless(w.dq[dn - 1 - mid], x0)) lo = mid + 1; else hi = mid;
+            if (qless(w.dq[mid], x0)) lo = mid + 1; else hi = mid;
         }
         int r = lo, run_r = lo, run_len = 0;
         for (int i = s0; i < s1; ++i) {
             const QEnt x = X[i];
-            while (r < dn && qless(w.dq[dn - 1 - r], x)) ++r;
+            while (r < dn && qless(w.dq[r], x)) ++r;
             out[i + r] = x;
             if (r != run_r) {
                 if (run_len) atomicAdd(&w.cnt[run_r], run_len);
@@ -189,7 +274,7 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
         if (run_len) atomicAdd(&w.cnt[run_r], run_len);
     }
     __syncwarp();
-    // delta element j (ascending) goes to j + sum_{r <= j} cnt[r]
+    // delta element j goes to j + #{main elements smaller} = j + sum_{r <= j} cnt[r]
     int carry = 0;
     for (int c0 = 0; c0 < dn; c0 += 32) {
         const int j = c0 + lane;
@@ -200,7 +285,7 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
             if (lane >= d) v += y;
         }
         v += carry;
-        if (j < dn) out[j + v] = w.dq[dn - 1 - j];
+        if (j < dn) out[j + v] = w.dq[j];
         carry = __shfl_sync(FULL, v, 31);
     }
     __syncwarp();
@@ -213,33 +298,22 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
     q.mcb = -1;
 }
 
-// Insert one entry into the delta (merging the delta into main first if it is full).
-__device__ void delta_insert(const Ws &w, Queue &q, const QEnt &e) {
-    const int lane = lane_id();
+__device__ __forceinline__ void delta_push(const Ws &w, Queue &q, const QEnt &e) {
     if (q.dn == w.dcap) merge_delta(w, q);
-    const int dn = q.dn;
-    // descending order: pos = #entries greater than e
-    const int pos = warp_prefix_count(dn, [&](int i) { return qless(e, w.dq[i]); });
-    for (int hi = dn; hi > pos; hi -= 32) {
-        const int lo = max(pos, hi - 32);
-        const int i = lo + lane;
-        QEnt v;
-        const bool act = i < hi;
-        if (act) v = w.dq[i];
-        __syncwarp();
-        if (act) w.dq[i + 1] = v;
-        __syncwarp();
-    }
-    if (lane == 0) w.dq[pos] = e;
+    if (lane_id() == 0) w.dq[q.dn] = e;
     __syncwarp();
-    q.dn = dn + 1;
+    if (q.dn == 0 || qless(e, q.dmin)) {
+        q.dmin = e;
+        q.dminpos = q.dn;
+    }
+    ++q.dn;
 }
 
 // Head of R_t (smallest (key, idx)); the queue must not be empty.  src: 0 main, 1 delta.
-__device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q, int &src) {
+__device__ __forceinline__ QEnt queue_head(Queue &q, int &src) {
     const int lane = lane_id();
-    bool have_m = q.mh < q.me;
-    QEnt hm, hd;
+    const bool have_m = q.mh < q.me;
+    QEnt hm;
     if (have_m) {
         if (q.mcb < 0 || q.mh < q.mcb || q.mh >= q.mcb + 32) {
             q.mcb = q.mh;
@@ -248,24 +322,29 @@ __device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q, int &src) {
         }
         hm = shfl_q(q.mc, q.mh - q.mcb);
     }
-    if (q.dn > 0) hd = w.dq[q.dn - 1];
-    if (have_m && (q.dn == 0 || qless(hm, hd))) {
+    if (have_m && (q.dn == 0 || qless(hm, q.dmin))) {
         src = 0;
         return hm;
     }
     src = 1;
-    return hd;
+    return q.dmin;
 }
 
-__device__ __forceinline__ void queue_pop(Queue &q, int src) {
-    if (src == 0) ++q.mh; else --q.dn;
+__device__ __forceinline__ void queue_pop(const Ws &w, Queue &q, int src) {
+    if (src == 0) {
+        ++q.mh;
+        return;
+    }
+    const int last = q.dn - 1;
+    if (lane_id() == 0 && q.dminpos != last) w.dq[q.dminpos] = w.dq[last];
+    __syncwarp();
+    q.dn = last;
+    if (q.dn > 0) delta_recompute_min(w, q);
 }
 
-// Arrival batch (ascending, global): becomes the main array if R_t is empty; a few entries go
-// into the delta one by one; a long batch is copied into the (emptied) delta in chunks, each
-// chunk merged into the main array.
+// Arrival batch (ascending run in global memory): becomes the main array if R_t is empty,
+// otherwise its entries go through the delta.
 __device__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
-    const int lane = lane_id();
     if (len <= 0) return;
     if (queue_empty(q)) {
         q.mq = run;
@@ -275,146 +354,212 @@ __device__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
         q.mcb = -1;
         return;
     }
-    int done = 0;
-    while (done < len) {
-        const int rem = len - done;
-        if (rem <= 8) {
-            for (int j = 0; j < rem; ++j) delta_insert(w, q, run[done + j]);
-            break;
-        }
-        if (q.dn > 0) merge_delta(w, q);
-        const int k = min(rem, w.dcap);
-        for (int j = lane; j < k; j += 32) w.dq[j] = run[done + k - 1 - j];  // descending
-        __syncwarp();
-        q.dn = k;
-        done += k;
-    }
+    for (int j = 0; j < len; ++j) delta_push(w, q, run[j]);
 }
 
 // ---------------------------------------------------------------------------------------------
-// Active set maintenance
+// Active set maintenance: one warp pass per change
 // ---------------------------------------------------------------------------------------------
-// Rebuild SB / PM for the current A entries relative to time base tb; also returns min F.
-__device__ void rebuild(const Ws &w, int A, int tb, int &SB0, int &nextF) {
+struct NewJob {
+    int e, f, b, p, id, k;
+};
+
+__device__ __forceinline__ void store_job(const Ws &w, int i, int e, int f, int b, int p, int id, int k) {
+    w.E[i] = e;
+    w.F[i] = f;
+    w.B[i] = b;
+    w.P[i] = p;
+    w.I[i] = id;
+    w.K[i] = k;
+}
+
+// SB, PM, SB0 and min F for the A entries (no dead entries), time base tb.
+__device__ void derive(const Ws &w, int A, int tb, int &SB0, int &nextF) {
     const int lane = lane_id();
     int carry = 0;
-    if (A > 0) {
-        for (int c0 = ((A - 1) >> 5) << 5; c0 >= 0; c0 -= 32) {
-            const int i = c0 + lane;
-            int x = (i < A) ? w.B[i] + tb : 0;
+    const int last = ((A - 1) / kChunk) * kChunk;
+    for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
+        const int base = cb + 4 * lane;
+        const int4 b4 = ld4(w.B, base);
+        const int bb[4] = {b4.x, b4.y, b4.z, b4.w};
+        int s[4];
+        int acc = 0;
 #pragma unroll
-            for (int d = 1; d < 32; d <<= 1) {
-                const int y = __shfl_down_sync(FULL, x, d);
-                if (lane + d < 32) x += y;
-            }
-            x += carry;
-            if (i < A) w.SB[i] = x;
-            carry = __shfl_sync(FULL, x, 0);
+        for (int j = 3; j >= 0; --j) {
+            acc += (base + j < A) ? bb[j] + tb : 0;
+            s[j] = acc;
         }
+        int tot;
+        const int after = excl_suffix_add(acc, tot) + carry;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (base + j < A) w.SB[base + j] = s[j] + after;
+        carry += tot;
     }
+    __syncwarp();
     if (lane == 0) {
         w.SB[A] = 0;
         w.PM[0] = INT_MIN;
     }
     SB0 = carry;
-    __syncwarp();
     int run = INT_MIN;
     int fmin = INT_MAX;
-    for (int c0 = 0; c0 < A; c0 += 32) {
-        const int i = c0 + lane;
-        int h = INT_MIN;
-        if (i < A) {
-            const int64_t e = int64_t(w.E[i]) - tb;
-            h = sat32(int64_t(w.SB[i]) + int64_t(A - i) * e + e);
-            fmin = min(fmin, w.F[i]);
-        }
+    for (int cb = 0; cb < A; cb += kChunk) {
+        const int base = cb + 4 * lane;
+        const int4 e4 = ld4(w.E, base), s4 = ld4(w.SB, base), f4 = ld4(w.F, base);
+        const int ee[4] = {e4.x, e4.y, e4.z, e4.w};
+        const int ss[4] = {s4.x, s4.y, s4.z, s4.w};
+        const int ff[4] = {f4.x, f4.y, f4.z, f4.w};
+        int m[4];
+        int mx = INT_MIN;
 #pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-            const int y = __shfl_up_sync(FULL, h, d);
-            if (lane >= d) h = max(h, y);
+        for (int j = 0; j < 4; ++j) {
+            int h = INT_MIN;
+            if (base + j < A) {
+                const int64_t e = int64_t(ee[j]) - tb;
+                h = sat32(int64_t(ss[j]) + int64_t(A - base - j) * e + e);
+                fmin = min(fmin, ff[j]);
+            }
+            mx = max(mx, h);
+            m[j] = mx;
         }
-        h = max(h, run);
-        if (i < A) w.PM[i + 1] = h;
-        run = __shfl_sync(FULL, h, 31);
+        const int before = max(excl_scan_max(mx), run);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (base + j < A) w.PM[base + j + 1] = max(before, m[j]);
+        run = max(run, __reduce_max_sync(FULL, mx));
     }
-    nextF = warp_min32(fmin);
+    nextF = __reduce_min_sync(FULL, fmin);
     __syncwarp();
 }
 
-// Remove entries marked dead (F < 0), keeping the order.  Returns the new size.
-__device__ int compact(const Ws &w, int A) {
+// Remove dead entries (F < 0), insert `nj` if ins, keep E ascending (new job after equal E),
+// then recompute the derived arrays.  Returns false if the capacity would be exceeded.
+__device__ bool rebuild(const Ws &w, int &A, int tb, bool ins, const NewJob &nj, int &SB0, int &nextF) {
     const int lane = lane_id();
-    int wpos = 0;
-    for (int c0 = 0; c0 < A; c0 += 32) {
-        const int i = c0 + lane;
-        const bool in = i < A;
-        int e = 0, f = -1, b = 0, p = 0, id = 0, k = 0;
-        if (in) {
-            f = w.F[i];
-            e = w.E[i];
-            b = w.B[i];
-            p = w.P[i];
-            id = w.I[i];
-            k = w.K[i];
+    if (A + (ins ? 1 : 0) <= kChunk) {
+        // single fused pass: every lane holds its 4 entries in registers before any store
+        const int base = 4 * lane;
+        const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
+        const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
+        const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
+        const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
+        const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+        bool lv[4];
+        int lc = 0, le = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            lv[j] = (base + j < A) && ff[j] >= 0;
+            lc += lv[j] ? 1 : 0;
+            le += (lv[j] && ins && ee[j] <= nj.e) ? 1 : 0;
         }
-        const bool live = in && f >= 0;
-        const unsigned bal = __ballot_sync(FULL, live);
-        const int dst = wpos + __popc(bal & ((1u << lane) - 1u));
+        int L;
+        const int off = excl_scan_add(lc, L);
+        const int pos = __reduce_add_sync(FULL, le);
         __syncwarp();
-        if (live) {
-            w.E[dst] = e;
-            w.F[dst] = f;
-            w.B[dst] = b;
-            w.P[dst] = p;
-            w.I[dst] = id;
-            w.K[dst] = k;
+        int qd = off;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (lv[j]) {
+                const int d = qd + ((ins && qd >= pos) ? 1 : 0);
+                store_job(w, d, ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
+                ++qd;
+            }
         }
+        if (ins && lane == 0) store_job(w, pos, nj.e, nj.f, nj.b, nj.p, nj.id, nj.k);
+        A = L + (ins ? 1 : 0);
         __syncwarp();
-        wpos += __popc(bal);
+    } else {
+        // compaction front to back (entries only move left), then the insertion shift
+        int wpos = 0;
+        for (int cb = 0; cb < A; cb += kChunk) {
+            const int base = cb + 4 * lane;
+            const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
+            const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
+            const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
+            const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
+            const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+            bool lv[4];
+            int lc = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                lv[j] = (base + j < A) && ff[j] >= 0;
+                lc += lv[j] ? 1 : 0;
+            }
+            int L;
+            const int off = excl_scan_add(lc, L);
+            __syncwarp();
+            int qd = wpos + off;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (lv[j]) store_job(w, qd++, ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
+            __syncwarp();
+            wpos += L;
+        }
+        A = wpos;
+        if (ins) {
+            if (A >= w.ca) return false;
+            const int pos = warp_prefix_count(A, [&](int i) { return w.E[i] <= nj.e; });
+            for (int hi = A; hi > pos; hi -= 32) {
+                const int lo = max(pos, hi - 32);
+                const int i = lo + lane;
+                const bool act = i < hi;
+                int ve = 0, vf = 0, vb = 0, vp = 0, vi = 0, vk = 0;
+                if (act) {
+                    ve = w.E[i];
+                    vf = w.F[i];
+                    vb = w.B[i];
+                    vp = w.P[i];
+                    vi = w.I[i];
+                    vk = w.K[i];
+                }
+                __syncwarp();
+                if (act) store_job(w, i + 1, ve, vf, vb, vp, vi, vk);
+                __syncwarp();
+            }
+            if (lane == 0) store_job(w, pos, nj.e, nj.f, nj.b, nj.p, nj.id, nj.k);
+            __syncwarp();
+            ++A;
+        }
     }
-    return wpos;
-}
-
-// Insert one active job keeping E ascending (after equal E).  Returns false if full.
-__device__ bool insert_active(const Ws &w, int &A, int e, int f, int b, int p, int id, int k) {
-    const int lane = lane_id();
-    if (A >= w.ca) return false;
-    const int pos = warp_prefix_count(A, [&](int i) { return w.E[i] <= e; });
-    for (int hi = A; hi > pos; hi -= 32) {
-        const int lo = max(pos, hi - 32);
-        const int i = lo + lane;
-        const bool act = i < hi;
-        int ve = 0, vf = 0, vb = 0, vp = 0, vi = 0, vk = 0;
-        if (act) {
-            ve = w.E[i];
-            vf = w.F[i];
-            vb = w.B[i];
-            vp = w.P[i];
-            vi = w.I[i];
-            vk = w.K[i];
-        }
-        __syncwarp();
-        if (act) {
-            w.E[i + 1] = ve;
-            w.F[i + 1] = vf;
-            w.B[i + 1] = vb;
-            w.P[i + 1] = vp;
-            w.I[i + 1] = vi;
-            w.K[i + 1] = vk;
-        }
-        __syncwarp();
-    }
-    if (lane == 0) {
-        w.E[pos] = e;
-        w.F[pos] = f;
-        w.B[pos] = b;
-        w.P[pos] = p;
-        w.I[pos] = id;
-        w.K[pos] = k;
-    }
-    __syncwarp();
-    ++A;
+    derive(w, A, tb, SB0, nextF);
     return true;
+}
+
+// First step tau in (t, tau_lim) at which the head candidate (prompt s, estimate L) fits, with the
+// active set unchanged; kBig if none.  In terms of y = tau + L - 1, the interval between active
+// endpoints (E[j-1], E[j]] has #{E < y} = j, and #{E <= y} = j below E[j] and the end of E[j]'s
+// group at y = E[j] (whose prefix maximum is PM[j+1]: within a group of equal E that lies at or
+// after tb the first entry has the largest H).  Conditions (1)-(3) give, per interval, a lower
+// bound on y from (2) and upper bounds from (1) and (3).
+__device__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int s, int L,
+                                  int64_t tau_lim) {
+    const int lane = lane_id();
+    const int64_t y0 = int64_t(t) + L - 1;
+    const int64_t ylim = tau_lim - 1 + L - 1;
+    const int64_t tau1 = tb + floor_div(M - s - 1 - SB0, A);  // (1)
+    const int64_t yup = min(ylim, tau1 + L - 1);
+    if (yup <= y0) return kBig;
+    const int64_t C2 = M - s - L - tb;
+    const int64_t C3 = M - s - L;
+    int64_t best = kBig;
+    for (int j = lane; j <= A; j += 32) {
+        const int64_t prev = (j == 0) ? -kBig : int64_t(w.E[j - 1]);
+        const int64_t cur = (j == A) ? kBig : int64_t(w.E[j]);
+        if (cur <= y0 || prev >= yup) continue;
+        const int64_t y3 = (A - j > 0) ? tb + floor_div(C3 - w.SB[j], A - j) : kBig;
+        const int64_t up = min(yup, y3);
+        const int64_t lo = max(prev + 1, y0 + 1);
+        const int64_t cand = max(lo, int64_t(w.PM[j]) - C2);
+        if (cand <= min(cur - 1, up)) best = min(best, cand);
+        if (j < A && cur > prev && cur >= y0 + 1 && cur <= up && int64_t(w.PM[j + 1]) - C2 <= cur)
+            best = min(best, cur);
+    }
+    // warp minimum: candidates lie in (y0, yup] and steps fit 31 bits, so y - y0 fits 32 bits
+    const unsigned off = (best == kBig) ? UINT_MAX : unsigned(best - y0);
+    const unsigned m = __reduce_min_sync(FULL, off);
+    if (m == UINT_MAX) return kBig;
+    return y0 + m - L + 1;
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -443,6 +588,7 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     q.mh = q.me = 0;
     q.mbuf = -1;
     q.dn = 0;
+    q.dminpos = 0;
     q.mcb = -1;
 
     int A = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
@@ -460,6 +606,8 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     bool pdirty = true;
     int64_t y_prev = 0;
     int hi = 0, lb = 0;
+    NewJob none;
+    none.e = none.f = none.b = none.p = none.id = none.k = 0;
 
     for (;;) {
         if (steps >= cap) {
@@ -471,8 +619,7 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
             int ae = ap;
             for (;;) {
                 const int i = ae + lane;
-                const bool ok = i < n && ra[i] <= t;
-                const unsigned b = __ballot_sync(FULL, ok);
+                const unsigned b = __ballot_sync(FULL, i < n && ra[i] <= t);
                 const int k = __popc(b);
                 ae += k;
                 if (k < 32) break;
@@ -495,35 +642,36 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
             int64_t need = int64_t(SB0) + int64_t(A) * (t - tb);
             if (need > M) {
                 while (need > M) {
-                    unsigned long long best = ~0ull;
-                    int bi = -1;
-                    for (int i = lane; i < A; i += 32) {
-                        if (w.F[i] >= 0) {
-                            const unsigned long long kk =
-                                (static_cast<unsigned long long>(static_cast<unsigned>(w.K[i])) << 32) |
-                                static_cast<unsigned>(w.I[i]);
-                            if (kk < best) {
-                                best = kk;
-                                bi = i;
+                    unsigned bk = UINT_MAX, bi = UINT_MAX;
+                    int bp = -1;
+                    for (int cb = 0; cb < A; cb += kChunk) {
+                        const int base = cb + 4 * lane;
+                        const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                        const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                        const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            if (base + j < A && ff[j] >= 0) {
+                                const unsigned k = unsigned(kk[j]), i = unsigned(ii[j]);
+                                if (k < bk || (k == bk && i < bi)) {
+                                    bk = k;
+                                    bi = i;
+                                    bp = base + j;
+                                }
                             }
                         }
                     }
-#pragma unroll
-                    for (int d = 16; d >= 1; d >>= 1) {
-                        const unsigned long long ob = __shfl_xor_sync(FULL, best, d);
-                        const int oi = __shfl_xor_sync(FULL, bi, d);
-                        if (ob < best) {
-                            best = ob;
-                            bi = oi;
-                        }
-                    }
-                    if (bi < 0) {
+                    const unsigned mk = __reduce_min_sync(FULL, bk);
+                    const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
+                    const unsigned ball = __ballot_sync(FULL, bp >= 0 && bk == mk && bi == mi);
+                    if (ball == 0) {
                         status = ST_STATE;
                         break;
                     }
-                    const int b = w.B[bi], p = w.P[bi], f = w.F[bi], k = w.K[bi], id = w.I[bi];
+                    const int pos = __shfl_sync(FULL, bp, __ffs(ball) - 1);
+                    const int b = w.B[pos], p = w.P[pos], f = w.F[pos], k = w.K[pos], id = w.I[pos];
                     __syncwarp();
-                    if (lane == 0) w.F[bi] = -1;
+                    if (lane == 0) w.F[pos] = -1;
                     __syncwarp();
                     QEnt e;
                     e.key = max(k, t - p);  // refined lower bound: max(estimate, tokens generated)
@@ -532,12 +680,11 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
                     e.o = f - p + 1;
                     need -= int64_t(b) + t;
                     ++nev;
-                    delta_insert(w, q, e);
+                    delta_push(w, q, e);
                 }
                 if (status != ST_OK) break;
-                A = compact(w, A);
                 tb = t;
-                rebuild(w, A, tb, SB0, nextF);
+                rebuild(w, A, tb, false, none, SB0, nextF);
                 hvalid = false;
                 pdirty = true;
             }
@@ -546,7 +693,7 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
         for (;;) {
             if (!hvalid) {
                 if (queue_empty(q)) break;
-                h = queue_head(w, q, hsrc);
+                h = queue_head(q, hsrc);
                 hvalid = true;
                 pdirty = true;
             }
@@ -564,37 +711,44 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
                 }
                 pdirty = false;
                 y_prev = y;
-                const int pm = w.PM[hi];
-                if (int64_t(pm) + h.s + 1 - dt > M) fits = false;
+                if (int64_t(w.PM[hi]) + h.s + 1 - dt > M) fits = false;
                 const int64_t v = int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb);
                 if (v + h.s + h.key > M) fits = false;
             } else if (fits) {
                 fits = int64_t(h.s) + h.key <= M;
             }
             if (!fits) break;
-            queue_pop(q, hsrc);
-            const int e = t + h.key - 1;
-            const int f = t + h.o - 1;
-            if (!insert_active(w, A, e, f, h.s - t + 1, t, h.idx, h.key)) {
+            queue_pop(w, q, hsrc);
+            NewJob nj;
+            nj.e = t + h.key - 1;
+            nj.f = t + h.o - 1;
+            nj.b = h.s - t + 1;
+            nj.p = t;
+            nj.id = h.idx;
+            nj.k = h.key;
+            if (A >= w.ca) {
                 status = kStatusCapacity;
                 break;
             }
             tb = t;
-            rebuild(w, A, tb, SB0, nextF);
+            if (!rebuild(w, A, tb, true, nj, SB0, nextF)) {
+                status = kStatusCapacity;
+                break;
+            }
             hvalid = false;
             pdirty = true;
         }
         if (status != ST_OK) break;
         // ---- S6: process the batch
-        const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
-        if (mem > M) {
-            status = ST_STATE;
-            break;
-        }
-        if (mem > peak) peak = mem;
-        rsteps += A;
-        ++steps;
         if (t == nextF) {
+            const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
+            if (mem > M) {
+                status = ST_STATE;
+                break;
+            }
+            if (mem > peak) peak = mem;
+            rsteps += A;
+            ++steps;
             int c = 0;
             for (int i = lane; i < A; i += 32) {
                 if (w.F[i] == t) {
@@ -603,18 +757,37 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
                     w.F[i] = -1;
                 }
             }
-            c = int(warp_sum64(c));
+            c = __reduce_add_sync(FULL, c);
             __syncwarp();
             sumC += int64_t(c) * (int64_t(t) + 1);
             makespan = int64_t(t) + 1;
             ndone += c;
-            A = compact(w, A);
             tb = t + 1;
-            rebuild(w, A, tb, SB0, nextF);
+            rebuild(w, A, tb, false, none, SB0, nextF);
             pdirty = true;
             if (ndone >= n) break;
+            ++t;
+        } else {
+            // steps t .. tau-1 change nothing: no completion before nextF, no arrival before
+            // next_a, (A_min) no overflow before tau_ov, and the head does not fit before tau_fit
+            int64_t tau = nextF;
+            if (ap < n) tau = min(tau, int64_t(next_a));
+            if (POL == P_AMIN && A > 0)
+                tau = min(tau, int64_t(tb) + floor_div(M - SB0, A) + 1);
+            tau = min(tau, int64_t(t) + (cap - steps));
+            if (tau > int64_t(t) + 1 && hvalid && A > 0)
+                tau = min(tau, first_fit_step(w, A, tb, SB0, M, t, h.s, h.key, tau));
+            const int64_t c = max(tau - int64_t(t), int64_t(1));
+            const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) + c - 1 - tb);
+            if (mem > M) {
+                status = ST_STATE;
+                break;
+            }
+            if (mem > peak) peak = mem;
+            rsteps += int64_t(A) * c;
+            steps += c;
+            t += int(c);
         }
-        ++t;
     }
     if (lane == 0) {
         r.status = status;
@@ -630,7 +803,7 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
 }
 
 template <int POL>
-__global__ void __launch_bounds__(256) k_run(RunParams P) {
+__global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
     const int wib = threadIdx.x >> 5;
@@ -650,136 +823,9 @@ __global__ void __launch_bounds__(256) k_run(RunParams P) {
     }
 }
 
-// ---------------------------------------------------------------------------------------------
-// Staging: validate, constants, sort by (a, key, idx)
-// ---------------------------------------------------------------------------------------------
-__device__ __forceinline__ bool stage_less(int aa, const QEnt &x, int ab, const QEnt &y) {
-    if (aa != ab) return aa < ab;
-    if (x.key != y.key) return x.key < y.key;
-    return x.idx < y.idx;
-}
-
-template <typename T>
-__device__ T block_reduce(T v, T *sh, bool is_max) {
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) {
-        const T o = __shfl_xor_sync(FULL, v, d);
-        v = is_max ? (o > v ? o : v) : v + o;
-    }
-    __syncthreads();
-    if (lane == 0) sh[wid] = v;
-    __syncthreads();
-    T acc = sh[0];
-    for (int i = 1; i < nw; ++i) acc = is_max ? (sh[i] > acc ? sh[i] : acc) : acc + sh[i];
-    return acc;
-}
-
-__global__ void __launch_bounds__(256) k_stage(StageParams S) {
-    __shared__ int64_t sh64[32];
-    const int inst = blockIdx.x;
-    const int64_t base = S.off[inst];
-    const int n = int(S.off[inst + 1] - base);
-    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, work = 0;
-    for (int j = threadIdx.x; j < n; j += blockDim.x) {
-        const int64_t g = base + j;
-        const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
-        if (s < 1 || a < 0 || l < 1 || l > o || o > u) bad_inval = 1;
-        if (int64_t(s) + o > S.M) bad_inf = 1;
-        if (S.policy == P_AMAX && int64_t(s) + u > S.M) bad_inf = 1;
-        const int key = (S.policy == P_AMAX) ? u : (S.policy == P_HSF ? o : l);
-        QEnt e;
-        e.key = key;
-        e.idx = j;
-        e.s = s;
-        e.o = o;
-        S.rec[g] = e;
-        S.rec_a[g] = a;
-        sum_a += a;
-        sum_o += o;
-        work += int64_t(s) * o + int64_t(o) * o / 2;
-    }
-    bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
-    bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
-    sum_a = block_reduce<int64_t>(sum_a, sh64, false);
-    sum_o = block_reduce<int64_t>(sum_o, sh64, false);
-    work = block_reduce<int64_t>(work, sh64, false);
-    int status = ST_OK;
-    if (bad_inval) status = ST_INVAL;
-    else if (bad_inf) status = ST_INFEASIBLE;
-    if (threadIdx.x == 0) {
-        InstInfo in;
-        in.base = base;
-        in.n = n;
-        in.status = status;
-        in.sum_a = sum_a;
-        in.cap = S.step_cap > 0 ? S.step_cap : 64 * (int64_t(n) + sum_o);
-        in.work = work;
-        S.info[inst] = in;
-    }
-    if (status != ST_OK || n <= 1) return;
-    __syncthreads();
-    // bitonic sort of [base, base + n) by (a, key, idx), padded virtually to a power of two
-    int N = 1;
-    while (N < n) N <<= 1;
-    QEnt *R = S.rec + base;
-    int32_t *RA = S.rec_a + base;
-    for (int k = 2; k <= N; k <<= 1) {
-        for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
-            const int half = k >> 1;
-            const int i = (p / half) * k + (p % half);
-            const int j = i ^ (k - 1);
-            if (j < n) {
-                const QEnt x = R[i], y = R[j];
-                const int ax = RA[i], ay = RA[j];
-                if (stage_less(ay, y, ax, x)) {
-                    R[i] = y;
-                    R[j] = x;
-                    RA[i] = ay;
-                    RA[j] = ax;
-                }
-            }
-        }
-        __syncthreads();
-        for (int d = k >> 2; d >= 1; d >>= 1) {
-            for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
-                const int i = (p / d) * 2 * d + (p % d);
-                const int j = i + d;
-                if (j < n) {
-                    const QEnt x = R[i], y = R[j];
-                    const int ax = RA[i], ay = RA[j];
-                    if (stage_less(ay, y, ax, x)) {
-                        R[i] = y;
-                        R[j] = x;
-                        RA[i] = ay;
-                        RA[j] = ax;
-                    }
-                }
-            }
-            __syncthreads();
-        }
-    }
-}
-
-__global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n) {
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= n) return;
-    const DevResult a = pol[i], b = ref[i];
-    double v = __longlong_as_double(0x7ff8000000000000ll);  // NaN
-    if (a.status == ST_OK && b.status == ST_OK && b.total_latency > 0)
-        v = double(a.total_latency) / double(b.total_latency);
-    out[i] = v;
-}
-
 }  // namespace
 
 size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
-
-cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
-    if (p.n_inst <= 0) return cudaSuccess;
-    k_stage<<<p.n_inst, 256, 0, st>>>(p);
-    return cudaGetLastError();
-}
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
     const void *fn = policy == P_AMAX ? (const void *)k_run<P_AMAX>
@@ -796,12 +842,6 @@ cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per
         case P_AMIN: k_run<P_AMIN><<<grid, block, smem_bytes, st>>>(p); break;
         default: k_run<P_HSF><<<grid, block, smem_bytes, st>>>(p); break;
     }
-    return cudaGetLastError();
-}
-
-cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st) {
-    if (n <= 0) return cudaSuccess;
-    k_ratio<<<(n + 255) / 256, 256, 0, st>>>(pol, ref, out, n);
     return cudaGetLastError();
 }
 

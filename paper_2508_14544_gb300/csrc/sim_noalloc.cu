@@ -41,12 +41,12 @@ constexpr int kNaDeltaCap = 256;
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Workspace bytes per warp for an active-set capacity of kNaMaxPerInstance (same formula as the
-// simulation kernel's carve: 6 x ca + 2 x (ca + 1) int32, 16-byte aligned, then the delta queue
+// simulation kernel's carve: 6 x ca + 2 x (ca + 4) int32, 16-byte aligned, then the delta queue
 // and its merge histogram).
 constexpr size_t ws_bytes_max() {
-    size_t b = size_t(6) * kNaMaxPerInstance * 4 + size_t(2) * (kNaMaxPerInstance + 1) * 4;
+    size_t b = size_t(6) * kNaMaxPerInstance * 4 + size_t(2) * (kNaMaxPerInstance + 4) * 4;
     b = (b + 15) & ~size_t(15);
-    b += size_t(kNaDeltaCap) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 1) * 4;
+    b += size_t(kNaDeltaCap) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 4) * 4;
     return (b + 15) & ~size_t(15);
 }
 
@@ -152,7 +152,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.info = d_info;
     p.res = reinterpret_cast<simgb::DevResult *>(results);
     p.completion = nullptr;
-    p.ca = int32_t(((std::max<int64_t>(n_max, 32) + 31) / 32) * 32);  // >= any active set: no fallback
+    p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
     p.dcap = kNaDeltaCap;
     p.use_smem = 0;
     p.gws = base + kOffWs;

@@ -1,0 +1,155 @@
+// Staging and result kernels of the batched scheduler simulator (sm_103a).
+//
+//   k_stage  - per instance (one CTA): validate the requests against the Section 2 model
+//              (1 <= l <= o <= u, s >= 1, a >= 0, s + o <= M; s + u <= M under A_max), compute the
+//              constants the simulation needs (sum of arrivals for TEL, the step cap), and sort
+//              the requests by (arrival step, policy key, index) so that every arrival batch is
+//              already in the order of the waiting set R_t (key u for Algorithm malb, l for
+//              Algorithms milb / milbrevise, o for Algorithm off).
+//   k_ratio  - per instance TEL(pi) / TEL(H-SF) in IEEE double (Definition cr).
+#include <climits>
+#include <cstdint>
+
+#include "sim_internal.h"
+
+namespace simgb {
+
+namespace {
+
+constexpr unsigned FULL = 0xffffffffu;
+enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
+enum { ST_OK = 0, ST_INVAL = -1, ST_INFEASIBLE = -2 };
+
+__device__ __forceinline__ bool stage_less(int aa, const QEnt &x, int ab, const QEnt &y) {
+    if (aa != ab) return aa < ab;
+    if (x.key != y.key) return x.key < y.key;
+    return x.idx < y.idx;
+}
+
+template <typename T>
+__device__ T block_reduce(T v, T *sh, bool is_max) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) {
+        const T o = __shfl_xor_sync(FULL, v, d);
+        v = is_max ? (o > v ? o : v) : v + o;
+    }
+    __syncthreads();
+    if (lane == 0) sh[wid] = v;
+    __syncthreads();
+    T acc = sh[0];
+    for (int i = 1; i < nw; ++i) acc = is_max ? (sh[i] > acc ? sh[i] : acc) : acc + sh[i];
+    return acc;
+}
+
+__global__ void __launch_bounds__(256) k_stage(StageParams S) {
+    __shared__ int64_t sh64[32];
+    const int inst = blockIdx.x;
+    const int64_t base = S.off[inst];
+    const int n = int(S.off[inst + 1] - base);
+    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, work = 0;
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+        const int64_t g = base + j;
+        const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
+        if (s < 1 || a < 0 || l < 1 || l > o || o > u) bad_inval = 1;
+        if (int64_t(s) + o > S.M) bad_inf = 1;
+        if (S.policy == P_AMAX && int64_t(s) + u > S.M) bad_inf = 1;
+        const int key = (S.policy == P_AMAX) ? u : (S.policy == P_HSF ? o : l);
+        QEnt e;
+        e.key = key;
+        e.idx = j;
+        e.s = s;
+        e.o = o;
+        S.rec[g] = e;
+        S.rec_a[g] = a;
+        sum_a += a;
+        sum_o += o;
+        work += int64_t(s) * o + int64_t(o) * o / 2;
+    }
+    bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
+    bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
+    sum_a = block_reduce<int64_t>(sum_a, sh64, false);
+    sum_o = block_reduce<int64_t>(sum_o, sh64, false);
+    work = block_reduce<int64_t>(work, sh64, false);
+    int status = ST_OK;
+    if (bad_inval) status = ST_INVAL;
+    else if (bad_inf) status = ST_INFEASIBLE;
+    if (threadIdx.x == 0) {
+        InstInfo in;
+        in.base = base;
+        in.n = n;
+        in.status = status;
+        in.sum_a = sum_a;
+        in.cap = S.step_cap > 0 ? S.step_cap : 64 * (int64_t(n) + sum_o);
+        in.work = work;
+        S.info[inst] = in;
+    }
+    if (status != ST_OK || n <= 1) return;
+    __syncthreads();
+    // bitonic sort of [base, base + n) by (a, key, idx), padded virtually to a power of two
+    int N = 1;
+    while (N < n) N <<= 1;
+    QEnt *R = S.rec + base;
+    int32_t *RA = S.rec_a + base;
+    for (int k = 2; k <= N; k <<= 1) {
+        for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
+            const int half = k >> 1;
+            const int i = (p / half) * k + (p % half);
+            const int j = i ^ (k - 1);
+            if (j < n) {
+                const QEnt x = R[i], y = R[j];
+                const int ax = RA[i], ay = RA[j];
+                if (stage_less(ay, y, ax, x)) {
+                    R[i] = y;
+                    R[j] = x;
+                    RA[i] = ay;
+                    RA[j] = ax;
+                }
+            }
+        }
+        __syncthreads();
+        for (int d = k >> 2; d >= 1; d >>= 1) {
+            for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
+                const int i = (p / d) * 2 * d + (p % d);
+                const int j = i + d;
+                if (j < n) {
+                    const QEnt x = R[i], y = R[j];
+                    const int ax = RA[i], ay = RA[j];
+                    if (stage_less(ay, y, ax, x)) {
+                        R[i] = y;
+                        R[j] = x;
+                        RA[i] = ay;
+                        RA[j] = ax;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
+__global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const DevResult a = pol[i], b = ref[i];
+    double v = __longlong_as_double(0x7ff8000000000000ll);  // NaN
+    if (a.status == ST_OK && b.status == ST_OK && b.total_latency > 0)
+        v = double(a.total_latency) / double(b.total_latency);
+    out[i] = v;
+}
+
+}  // namespace
+
+cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
+    if (p.n_inst <= 0) return cudaSuccess;
+    k_stage<<<p.n_inst, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_ratio<<<(n + 255) / 256, 256, 0, st>>>(pol, ref, out, n);
+    return cudaGetLastError();
+}
+
+}  // namespace simgb
