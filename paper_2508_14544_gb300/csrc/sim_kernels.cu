@@ -1,4 +1,4 @@
-// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy>.
+// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared>.
 //
 // One warp simulates one instance at a time (persistent warps pull instance ids from a work
 // queue).  Each step follows the paper's algorithms:
@@ -6,8 +6,8 @@
 //   S3  A_min only (Algorithm milb): if the next step of the active set would exceed M, cancel
 //       jobs in ascending (estimate, index) order until it fits; each cancelled job's estimate
 //       becomes max(estimate, tokens generated) and it re-enters R_t in the same step;
-//   S5  admit the head of R_t (sorted by (key, index)) while eq. Constraint holds at every future
-//       step: the largest feasible prefix (Algorithms malb / milb / off);
+//   S5  admit the largest prefix of R_t (sorted by (key, index)) for which eq. Constraint holds at
+//       every future step (Algorithms malb / milb / off);
 //   S6  process the batch: one token per member, the step's memory sum(s + tokens) (eq.
 //       constraintM), completions, TEL (eq. latency).
 //
@@ -29,7 +29,12 @@
 //   (3) V(y) + s + L <= M,  y = t + L - 1                (its own last step),
 // so a step in which nothing changes costs O(1), and a run of such steps is processed in closed
 // form up to the next event (completion, arrival, A_min overflow, or the first step at which
-// the head fits, found by scanning the segments between active endpoints).
+// the head fits, found by scanning the segments between active endpoints).  When the head fits,
+// the whole admitted prefix is found at once on a window of the first 32 entries of R_t: with
+// CS[k] = sum_{m<k} (s_m + 1), prefix k adds CS[k] - CS[r] + (k - r)(x - t) to the projected
+// memory at step x, where r counts the window entries that end before x; each point (x = t,
+// every active endpoint, every window entry's endpoint) yields the first k at which it exceeds
+// M, and the admitted count is the minimum of those, less one.
 #include <climits>
 #include <cstdint>
 
@@ -43,6 +48,7 @@ constexpr unsigned FULL = 0xffffffffu;
 enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
 enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
 constexpr int kChunk = 128;  // active-set entries per warp pass (4 per lane)
+constexpr int kWin = 32;     // admission window (one candidate per lane)
 constexpr int64_t kBig = int64_t(1) << 60;
 
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
@@ -60,15 +66,6 @@ __device__ __forceinline__ int64_t floor_div(int64_t a, int64_t b) {  // b > 0
     int64_t q = a / b;
     if ((a % b != 0) && (a < 0)) --q;
     return q;
-}
-
-__device__ __forceinline__ QEnt shfl_q(const QEnt &q, int src) {
-    QEnt r;
-    r.key = __shfl_sync(FULL, q.key, src);
-    r.idx = __shfl_sync(FULL, q.idx, src);
-    r.s = __shfl_sync(FULL, q.s, src);
-    r.o = __shfl_sync(FULL, q.o, src);
-    return r;
 }
 
 // Exclusive prefix sum over lanes; total = sum over all lanes.
@@ -110,7 +107,7 @@ __device__ __forceinline__ int excl_scan_max(int v) {
     return lane == 0 ? INT_MIN : ex;
 }
 
-// Number of leading positions i in [0, len) with pred(i) true (pred true on a prefix).
+// Number of leading positions i in [0, len) with pred(i) true (pred true on a prefix); warp-wide.
 template <class Pred>
 __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
     if (len <= 0) return 0;
@@ -131,14 +128,28 @@ __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
     return cnt;
 }
 
+// The same, computed by one lane alone (binary search).
+template <class Pred>
+__device__ __forceinline__ int lane_prefix_count(int len, Pred pred) {
+    int lo = 0, hi = len;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (pred(mid)) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
 // ---------------------------------------------------------------------------------------------
 // Per-warp workspace
 // ---------------------------------------------------------------------------------------------
 struct Ws {
     int32_t *E, *F, *B, *P, *I, *K;  // active set, capacity ca (multiple of kChunk), 16-byte aligned
     int32_t *SB, *PM;                // ca + 4
-    QEnt *dq;                        // delta queue, dcap entries (power of two), unsorted
+    QEnt *dq;                        // delta queue, dcap entries, sorted DESCENDING (head = dq[dn-1])
+    QEnt *win;                       // admission window, kWin entries in (key, idx) order
+    QEnt *mc;                        // cached head of the main queue, kWin entries
     int32_t *cnt;                    // dcap + 4 (merge histogram)
+    int32_t *wkey, *wcs, *wsrc;      // window keys, prefix sums CS[0..kWin], sources (0 main, 1 delta)
     QEnt *mb0, *mb1;                 // global ping-pong main-queue buffers
     int32_t ca, dcap;
 };
@@ -146,11 +157,12 @@ struct Ws {
 __host__ __device__ inline size_t ws_bytes_impl(int ca, int dcap) {
     size_t b = size_t(6) * ca * sizeof(int32_t) + size_t(2) * (ca + 4) * sizeof(int32_t);
     b = (b + 15) & ~size_t(15);
-    b += size_t(dcap) * sizeof(QEnt) + size_t(dcap + 4) * sizeof(int32_t);
+    b += size_t(dcap + 2 * kWin) * sizeof(QEnt);
+    b += size_t(dcap + 4) * sizeof(int32_t) + size_t(kWin + kWin + 4 + kWin) * sizeof(int32_t);
     return (b + 15) & ~size_t(15);
 }
 
-__device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
+__device__ __forceinline__ Ws carve_ws(unsigned char *base, int ca, int dcap) {
     Ws w;
     int32_t *p = reinterpret_cast<int32_t *>(base);
     w.E = p; p += ca;
@@ -164,7 +176,12 @@ __device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
     size_t off = size_t(reinterpret_cast<unsigned char *>(p) - base);
     off = (off + 15) & ~size_t(15);
     w.dq = reinterpret_cast<QEnt *>(base + off);
-    w.cnt = reinterpret_cast<int32_t *>(w.dq + dcap);
+    w.win = w.dq + dcap;
+    w.mc = w.win + kWin;
+    w.cnt = reinterpret_cast<int32_t *>(w.mc + kWin);
+    w.wkey = w.cnt + dcap + 4;
+    w.wcs = w.wkey + kWin;
+    w.wsrc = w.wcs + kWin + 4;
     w.ca = ca;
     w.dcap = dcap;
     return w;
@@ -173,77 +190,34 @@ __device__ inline Ws carve_ws(unsigned char *base, int ca, int dcap) {
 __device__ __forceinline__ int4 ld4(const int32_t *a, int i) { return *reinterpret_cast<const int4 *>(a + i); }
 
 // ---------------------------------------------------------------------------------------------
-// Waiting set R_t: a sorted main array in global memory [mh, me) (lane-cached head) plus an
-// unsorted delta array in the workspace with its minimum cached.  A full delta is sorted (warp
-// bitonic sort) and merged into the main array.  Order: (key, idx).
+// Waiting set R_t: a sorted main array in global memory [mh, me) (its first kWin entries cached
+// in the workspace) plus a small sorted delta array (descending, so the head is the last
+// entry).  Together they hold R_t in (key, idx) order.  Inserts go to the delta; a full delta is
+// merged into the main array.
 // ---------------------------------------------------------------------------------------------
 struct Queue {
     const QEnt *mq;  // main array (global, ascending); may point into the staged records
     int mh, me;      // head / end
     int mbuf;        // -1: mq is read-only staged data; 0/1: ping-pong buffer in use
     int dn;          // delta size
-    int dminpos;     // position of the delta minimum
-    QEnt dmin;       // delta minimum
-    int mcb;         // main head cache base (lane l caches mq[mcb + l]), -1 invalid
-    QEnt mc;         // this lane's cached main entry
+    int mcb;         // main cache base: w.mc[i] = mq[mcb + i]; -1 invalid
 };
 
 __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.me && q.dn == 0; }
 
-__device__ void delta_recompute_min(const Ws &w, Queue &q) {
-    const int lane = lane_id();
-    unsigned bk = UINT_MAX, bi = UINT_MAX;
-    int bp = -1;
-    for (int j = lane; j < q.dn; j += 32) {
-        const QEnt e = w.dq[j];
-        const unsigned k = unsigned(e.key), i = unsigned(e.idx);
-        if (k < bk || (k == bk && i < bi)) {
-            bk = k;
-            bi = i;
-            bp = j;
-        }
-    }
-    const unsigned mk = __reduce_min_sync(FULL, bk);
-    const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
-    const unsigned ball = __ballot_sync(FULL, bp >= 0 && bk == mk && bi == mi);
-    const int src = ball ? __ffs(ball) - 1 : 0;
-    q.dminpos = __shfl_sync(FULL, bp, src);
-    if (q.dn > 0) q.dmin = w.dq[q.dminpos];
-}
-
-// Sort the delta ascending in place (bitonic network over dcap entries, padded with +inf).
-__device__ void delta_sort(const Ws &w, int dn) {
-    const int lane = lane_id();
-    const int D = w.dcap;
-    QEnt inf;
-    inf.key = INT_MAX;
-    inf.idx = INT_MAX;
-    inf.s = 0;
-    inf.o = 0;
-    for (int j = dn + lane; j < D; j += 32) w.dq[j] = inf;
+// Make w.mc hold mq[mh .. mh + kWin).
+__device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
+    if (q.mcb == q.mh) return;
+    const int i = q.mh + lane_id();
+    if (i < q.me) w.mc[lane_id()] = q.mq[i];
     __syncwarp();
-    for (int k = 2; k <= D; k <<= 1) {
-        for (int j = k >> 1; j > 0; j >>= 1) {
-            for (int p = lane; p < (D >> 1); p += 32) {
-                const int i = (p / j) * 2 * j + (p % j);
-                const int l = i + j;
-                const QEnt a = w.dq[i], b = w.dq[l];
-                const bool asc = (i & k) == 0;
-                if (qless(b, a) == asc) {
-                    w.dq[i] = b;
-                    w.dq[l] = a;
-                }
-            }
-            __syncwarp();
-        }
-    }
+    q.mcb = q.mh;
 }
 
 // Merge the delta into the main array (into the other ping-pong buffer).
-__device__ void merge_delta(const Ws &w, Queue &q) {
+__device__ __forceinline__ void merge_delta(const Ws &w, Queue &q) {
     const int lane = lane_id();
     const int dn = q.dn;
-    delta_sort(w, dn);
     const int nx = q.me - q.mh;
     QEnt *out = (q.mbuf == 0) ? w.mb1 : w.mb0;
     const QEnt *X = q.mq + q.mh;
@@ -254,15 +228,11 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
     const int s1 = min(s0 + c, nx);
     if (s0 < s1) {
         const QEnt x0 = X[s0];
-        int lo = 0, hi = dn;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (qless(w.dq[mid], x0)) lo = mid + 1; else hi = mid;
-        }
-        int r = lo, run_r = lo, run_len = 0;
+        int r = lane_prefix_count(dn, [&](int m) { return qless(w.dq[dn - 1 - m], x0); });
+        int run_r = r, run_len = 0;
         for (int i = s0; i < s1; ++i) {
             const QEnt x = X[i];
-            while (r < dn && qless(w.dq[r], x)) ++r;
+            while (r < dn && qless(w.dq[dn - 1 - r], x)) ++r;
             out[i + r] = x;
             if (r != run_r) {
                 if (run_len) atomicAdd(&w.cnt[run_r], run_len);
@@ -274,7 +244,7 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
         if (run_len) atomicAdd(&w.cnt[run_r], run_len);
     }
     __syncwarp();
-    // delta element j goes to j + #{main elements smaller} = j + sum_{r <= j} cnt[r]
+    // delta element j (ascending) goes to j + #{main entries smaller} = j + sum_{r <= j} cnt[r]
     int carry = 0;
     for (int c0 = 0; c0 < dn; c0 += 32) {
         const int j = c0 + lane;
@@ -285,7 +255,7 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
             if (lane >= d) v += y;
         }
         v += carry;
-        if (j < dn) out[j + v] = w.dq[j];
+        if (j < dn) out[j + v] = w.dq[dn - 1 - j];
         carry = __shfl_sync(FULL, v, 31);
     }
     __syncwarp();
@@ -298,53 +268,49 @@ __device__ void merge_delta(const Ws &w, Queue &q) {
     q.mcb = -1;
 }
 
-__device__ __forceinline__ void delta_push(const Ws &w, Queue &q, const QEnt &e) {
+// Insert one entry into the delta (merging the delta into main first if it is full).
+__device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &e) {
+    const int lane = lane_id();
     if (q.dn == w.dcap) merge_delta(w, q);
-    if (lane_id() == 0) w.dq[q.dn] = e;
-    __syncwarp();
-    if (q.dn == 0 || qless(e, q.dmin)) {
-        q.dmin = e;
-        q.dminpos = q.dn;
+    const int dn = q.dn;
+    const int pos = warp_prefix_count(dn, [&](int i) { return qless(e, w.dq[i]); });  // #entries > e
+    for (int hi = dn; hi > pos; hi -= 32) {
+        const int lo = max(pos, hi - 32);
+        const int i = lo + lane;
+        QEnt v;
+        const bool act = i < hi;
+        if (act) v = w.dq[i];
+        __syncwarp();
+        if (act) w.dq[i + 1] = v;
+        __syncwarp();
     }
-    ++q.dn;
+    if (lane == 0) w.dq[pos] = e;
+    __syncwarp();
+    q.dn = dn + 1;
 }
 
-// Head of R_t (smallest (key, idx)); the queue must not be empty.  src: 0 main, 1 delta.
-__device__ __forceinline__ QEnt queue_head(Queue &q, int &src) {
-    const int lane = lane_id();
+// Head of R_t (smallest (key, idx)); the queue must not be empty.
+__device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q) {
     const bool have_m = q.mh < q.me;
     QEnt hm;
     if (have_m) {
-        if (q.mcb < 0 || q.mh < q.mcb || q.mh >= q.mcb + 32) {
-            q.mcb = q.mh;
-            const int i = q.mcb + lane;
-            if (i < q.me) q.mc = q.mq[i];
+        if (q.mcb < 0 || q.mh < q.mcb || q.mh >= q.mcb + kWin) {
+            q.mcb = -1;
+            main_cache_at_head(w, q);
         }
-        hm = shfl_q(q.mc, q.mh - q.mcb);
+        hm = w.mc[q.mh - q.mcb];
     }
-    if (have_m && (q.dn == 0 || qless(hm, q.dmin))) {
-        src = 0;
-        return hm;
+    if (q.dn > 0) {
+        const QEnt hd = w.dq[q.dn - 1];
+        if (!have_m || qless(hd, hm)) return hd;
     }
-    src = 1;
-    return q.dmin;
+    return hm;
 }
 
-__device__ __forceinline__ void queue_pop(const Ws &w, Queue &q, int src) {
-    if (src == 0) {
-        ++q.mh;
-        return;
-    }
-    const int last = q.dn - 1;
-    if (lane_id() == 0 && q.dminpos != last) w.dq[q.dminpos] = w.dq[last];
-    __syncwarp();
-    q.dn = last;
-    if (q.dn > 0) delta_recompute_min(w, q);
-}
-
-// Arrival batch (ascending run in global memory): becomes the main array if R_t is empty,
-// otherwise its entries go through the delta.
-__device__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
+// Arrival batch (ascending run in global memory): becomes the main array if R_t is empty; a few
+// entries go into the delta one by one; a long batch is copied into the emptied delta in chunks.
+__device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
+    const int lane = lane_id();
     if (len <= 0) return;
     if (queue_empty(q)) {
         q.mq = run;
@@ -354,16 +320,55 @@ __device__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
         q.mcb = -1;
         return;
     }
-    for (int j = 0; j < len; ++j) delta_push(w, q, run[j]);
+    int done = 0;
+    while (done < len) {
+        const int rem = len - done;
+        if (rem <= 8) {
+            for (int j = 0; j < rem; ++j) delta_insert(w, q, run[done + j]);
+            break;
+        }
+        if (q.dn > 0) merge_delta(w, q);
+        const int k = min(rem, w.dcap);
+        for (int j = lane; j < k; j += 32) w.dq[j] = run[done + k - 1 - j];  // descending
+        __syncwarp();
+        q.dn = k;
+        done += k;
+    }
+}
+
+// First kWin entries of R_t in (key, idx) order into w.win / w.wsrc; returns how many.
+__device__ __forceinline__ int build_window(const Ws &w, Queue &q) {
+    const int lane = lane_id();
+    const int nmain = q.me - q.mh;
+    if (nmain > 0) main_cache_at_head(w, q);
+    const int nm = min(kWin, max(nmain, 0));
+    const int dn = q.dn;
+    const int nd = min(kWin, dn);
+    if (lane < nm) {
+        const QEnt x = w.mc[lane];
+        const int r = lane_prefix_count(dn, [&](int m) { return qless(w.dq[dn - 1 - m], x); });
+        const int pos = lane + r;
+        if (pos < kWin) {
+            w.win[pos] = x;
+            w.wsrc[pos] = 0;
+        }
+    }
+    if (lane < nd) {
+        const QEnt y = w.dq[dn - 1 - lane];
+        const int c = lane_prefix_count(nm, [&](int m) { return qless(w.mc[m], y); });
+        const int pos = lane + c;
+        if (pos < kWin) {
+            w.win[pos] = y;
+            w.wsrc[pos] = 1;
+        }
+    }
+    __syncwarp();
+    return min(kWin, max(nmain, 0) + dn);
 }
 
 // ---------------------------------------------------------------------------------------------
-// Active set maintenance: one warp pass per change
+// Active set maintenance
 // ---------------------------------------------------------------------------------------------
-struct NewJob {
-    int e, f, b, p, id, k;
-};
-
 __device__ __forceinline__ void store_job(const Ws &w, int i, int e, int f, int b, int p, int id, int k) {
     w.E[i] = e;
     w.F[i] = f;
@@ -374,7 +379,7 @@ __device__ __forceinline__ void store_job(const Ws &w, int i, int e, int f, int 
 }
 
 // SB, PM, SB0 and min F for the A entries (no dead entries), time base tb.
-__device__ void derive(const Ws &w, int A, int tb, int &SB0, int &nextF) {
+__device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int &nextF) {
     const int lane = lane_id();
     int carry = 0;
     const int last = ((A - 1) / kChunk) * kChunk;
@@ -433,97 +438,135 @@ __device__ void derive(const Ws &w, int A, int tb, int &SB0, int &nextF) {
     __syncwarp();
 }
 
-// Remove dead entries (F < 0), insert `nj` if ins, keep E ascending (new job after equal E),
-// then recompute the derived arrays.  Returns false if the capacity would be exceeded.
-__device__ bool rebuild(const Ws &w, int &A, int tb, bool ins, const NewJob &nj, int &SB0, int &nextF) {
+// Remove the entries marked dead (F < 0), keeping the order; entries only move left.
+__device__ __forceinline__ void compact(const Ws &w, int &A) {
     const int lane = lane_id();
-    if (A + (ins ? 1 : 0) <= kChunk) {
-        // single fused pass: every lane holds its 4 entries in registers before any store
-        const int base = 4 * lane;
+    int wpos = 0;
+    for (int cb = 0; cb < A; cb += kChunk) {
+        const int base = cb + 4 * lane;
         const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
         const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
         const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
         const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
         const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
         bool lv[4];
-        int lc = 0, le = 0;
+        int lc = 0;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             lv[j] = (base + j < A) && ff[j] >= 0;
             lc += lv[j] ? 1 : 0;
-            le += (lv[j] && ins && ee[j] <= nj.e) ? 1 : 0;
         }
         int L;
         const int off = excl_scan_add(lc, L);
-        const int pos = __reduce_add_sync(FULL, le);
         __syncwarp();
-        int qd = off;
+        int qd = wpos + off;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (lv[j]) store_job(w, qd++, ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
+        __syncwarp();
+        wpos += L;
+    }
+    A = wpos;
+}
+
+// Insert the K window entries admitted at step t (lane m < K holds entry m, ascending E) into the
+// compact active set, keeping E ascending (new entries after equal old ones).  Entries only move
+// right, so chunks are processed from the back.  Returns false if the capacity is exceeded.
+__device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t, const QEnt &mine) {
+    const int lane = lane_id();
+    if (A + K > w.ca) return false;
+    const int ne = t + mine.key - 1;
+    // destination of new entry m: m + #{old E <= E_m}
+    const int posm = (lane < K) ? lane + lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; }) : 0;
+    const int last = ((A - 1) / kChunk) * kChunk;
+    for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
+        const int base = cb + 4 * lane;
+        const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
+        const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
+        const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
+        const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
+        const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+        int sh[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            if (lv[j]) {
-                const int d = qd + ((ins && qd >= pos) ? 1 : 0);
-                store_job(w, d, ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
-                ++qd;
-            }
+            // #{new m < K: E_m < E_j},  E_m = t + key_m - 1 ascending in m
+            const int lim = ee[j] - t + 1;  // E_m < E_j  <=>  key_m < lim
+            sh[j] = (base + j < A) ? lane_prefix_count(K, [&](int m) { return w.wkey[m] < lim; }) : 0;
         }
-        if (ins && lane == 0) store_job(w, pos, nj.e, nj.f, nj.b, nj.p, nj.id, nj.k);
-        A = L + (ins ? 1 : 0);
         __syncwarp();
-    } else {
-        // compaction front to back (entries only move left), then the insertion shift
-        int wpos = 0;
-        for (int cb = 0; cb < A; cb += kChunk) {
-            const int base = cb + 4 * lane;
-            const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
-            const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
-            const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
-            const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
-            const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-            bool lv[4];
-            int lc = 0;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                lv[j] = (base + j < A) && ff[j] >= 0;
-                lc += lv[j] ? 1 : 0;
-            }
-            int L;
-            const int off = excl_scan_add(lc, L);
-            __syncwarp();
-            int qd = wpos + off;
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-                if (lv[j]) store_job(w, qd++, ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
-            __syncwarp();
-            wpos += L;
+        for (int j = 0; j < 4; ++j)
+            if (base + j < A) store_job(w, base + j + sh[j], ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
+        __syncwarp();
+    }
+    if (lane < K) store_job(w, posm, ne, t + mine.o - 1, mine.s - t + 1, t, mine.idx, mine.key);
+    __syncwarp();
+    A += K;
+    return true;
+}
+
+// Largest admissible prefix of the window at step t (see the file comment).  Lane m holds window
+// entry m (m < W); the active set is compact with derived arrays for time base tb.
+__device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int W,
+                                                 const QEnt &mine) {
+    const int lane = lane_id();
+    // prefix sums CS[k] = sum_{m<k} (s_m + 1)
+    int tot;
+    const int add = lane < W ? mine.s + 1 : 0;
+    const int ex = excl_scan_add(add, tot);
+    const int incl = ex + add;
+    if (lane < W) {
+        w.wkey[lane] = mine.key;
+        w.wcs[lane + 1] = incl;
+    }
+    if (lane == 0) w.wcs[0] = 0;
+    __syncwarp();
+    const int64_t dt = int64_t(t) - tb;
+    const int64_t need = int64_t(SB0) + int64_t(A) * dt;
+    const int64_t csW = tot;
+    // the coming step (x = t): every window entry adds s + 1
+    const unsigned ball = __ballot_sync(FULL, lane < W && need + incl > M);
+    int phi = ball ? __ffs(ball) : W + 1;
+    // active endpoints x = E_j >= t
+    for (int j = lane; j < A; j += 32) {
+        const int ej = w.E[j];
+        if (ej < t) continue;
+        const int64_t d = int64_t(ej) - t;
+        const int64_t v0 = int64_t(w.SB[j]) + int64_t(A - j) * (int64_t(ej) - tb);
+        if (v0 + csW + int64_t(W) * d <= M) continue;
+        if (v0 > M) {
+            phi = 0;
+            continue;
         }
-        A = wpos;
-        if (ins) {
-            if (A >= w.ca) return false;
-            const int pos = warp_prefix_count(A, [&](int i) { return w.E[i] <= nj.e; });
-            for (int hi = A; hi > pos; hi -= 32) {
-                const int lo = max(pos, hi - 32);
-                const int i = lo + lane;
-                const bool act = i < hi;
-                int ve = 0, vf = 0, vb = 0, vp = 0, vi = 0, vk = 0;
-                if (act) {
-                    ve = w.E[i];
-                    vf = w.F[i];
-                    vb = w.B[i];
-                    vp = w.P[i];
-                    vi = w.I[i];
-                    vk = w.K[i];
-                }
-                __syncwarp();
-                if (act) store_job(w, i + 1, ve, vf, vb, vp, vi, vk);
-                __syncwarp();
+        const int r = lane_prefix_count(W, [&](int m) { return int64_t(w.wkey[m]) <= d; });
+        if (r >= W) continue;
+        const int64_t base = v0 - w.wcs[r] - int64_t(r) * d;
+        if (base + csW + int64_t(W) * d <= M) continue;
+        int lo = r + 1, hi = W;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (base + w.wcs[mid] + int64_t(mid) * d > M) hi = mid; else lo = mid + 1;
+        }
+        phi = min(phi, lo);
+    }
+    // the window entries' own last steps x = t + key_m - 1
+    if (lane < W) {
+        const int64_t d = int64_t(mine.key) - 1;
+        const int64_t y = int64_t(t) + d;
+        const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
+        const int64_t av = int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb);
+        const int64_t base = av - ex - int64_t(lane) * d;  // ex = CS[lane]
+        if (base + csW + int64_t(W) * d > M) {
+            int lo = lane + 1, hi = W;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (base + w.wcs[mid] + int64_t(mid) * d > M) hi = mid; else lo = mid + 1;
             }
-            if (lane == 0) store_job(w, pos, nj.e, nj.f, nj.b, nj.p, nj.id, nj.k);
-            __syncwarp();
-            ++A;
+            phi = min(phi, lo);
         }
     }
-    derive(w, A, tb, SB0, nextF);
-    return true;
+    phi = __reduce_min_sync(FULL, phi);
+    return min(max(phi - 1, 0), W);
 }
 
 // First step tau in (t, tau_lim) at which the head candidate (prompt s, estimate L) fits, with the
@@ -532,8 +575,8 @@ __device__ bool rebuild(const Ws &w, int &A, int tb, bool ins, const NewJob &nj,
 // group at y = E[j] (whose prefix maximum is PM[j+1]: within a group of equal E that lies at or
 // after tb the first entry has the largest H).  Conditions (1)-(3) give, per interval, a lower
 // bound on y from (2) and upper bounds from (1) and (3).
-__device__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int s, int L,
-                                  int64_t tau_lim) {
+__device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int s,
+                                                  int L, int64_t tau_lim) {
     const int lane = lane_id();
     const int64_t y0 = int64_t(t) + L - 1;
     const int64_t ylim = tau_lim - 1 + L - 1;
@@ -566,7 +609,7 @@ __device__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M
 // One instance, simulated by one warp.  All lanes hold identical copies of the scalar state.
 // ---------------------------------------------------------------------------------------------
 template <int POL>
-__device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
+__device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     const int lane = lane_id();
     const InstInfo info = P.info[inst];
     DevResult r;
@@ -588,10 +631,14 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     q.mh = q.me = 0;
     q.mbuf = -1;
     q.dn = 0;
-    q.dminpos = 0;
     q.mcb = -1;
 
     int A = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
+    if (lane == 0) {  // derived arrays of the empty active set (the workspace is reused)
+        w.SB[0] = 0;
+        w.PM[0] = INT_MIN;
+    }
+    __syncwarp();
     int t = ra[0];
     int ap = 0;
     int next_a = t;
@@ -602,12 +649,9 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
 
     bool hvalid = false;
     QEnt h;
-    int hsrc = 0;
     bool pdirty = true;
     int64_t y_prev = 0;
     int hi = 0, lb = 0;
-    NewJob none;
-    none.e = none.f = none.b = none.p = none.id = none.k = 0;
 
     for (;;) {
         if (steps >= cap) {
@@ -680,23 +724,25 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
                     e.o = f - p + 1;
                     need -= int64_t(b) + t;
                     ++nev;
-                    delta_push(w, q, e);
+                    delta_insert(w, q, e);
                 }
                 if (status != ST_OK) break;
+                compact(w, A);
                 tb = t;
-                rebuild(w, A, tb, false, none, SB0, nextF);
+                derive(w, A, tb, SB0, nextF);
                 hvalid = false;
                 pdirty = true;
             }
         }
-        // ---- S4/S5: admit the head of R_t while it fits (largest feasible prefix)
+        // ---- S4/S5: admit the largest feasible prefix of R_t
         for (;;) {
             if (!hvalid) {
                 if (queue_empty(q)) break;
-                h = queue_head(q, hsrc);
+                h = queue_head(w, q);
                 hvalid = true;
                 pdirty = true;
             }
+            // quick test of the head alone (the prefix of length one)
             const int64_t dt = int64_t(t) - tb;
             const int64_t need = int64_t(SB0) + int64_t(A) * dt;
             bool fits = need + h.s + 1 <= M;
@@ -718,25 +764,37 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
                 fits = int64_t(h.s) + h.key <= M;
             }
             if (!fits) break;
-            queue_pop(w, q, hsrc);
-            NewJob nj;
-            nj.e = t + h.key - 1;
-            nj.f = t + h.o - 1;
-            nj.b = h.s - t + 1;
-            nj.p = t;
-            nj.id = h.idx;
-            nj.k = h.key;
-            if (A >= w.ca) {
+            // the head fits: find the whole admissible prefix on the window
+            const int W = build_window(w, q);
+            QEnt mine;
+            mine.key = mine.idx = mine.s = mine.o = 0;
+            int msrc = 0;
+            if (lane < W) {
+                mine = w.win[lane];
+                msrc = w.wsrc[lane];
+            }
+            const int Kadm = admissible_prefix(w, A, tb, SB0, M, t, W, mine);
+            if (Kadm <= 0) {
+                status = ST_STATE;  // the head test and the window disagree: internal error
+                break;
+            }
+            const int cm = __popc(__ballot_sync(FULL, lane < Kadm && msrc == 0));
+            q.mh += cm;
+            q.dn -= Kadm - cm;
+            if (!insert_window(w, A, Kadm, t, mine)) {
                 status = kStatusCapacity;
                 break;
             }
             tb = t;
-            if (!rebuild(w, A, tb, true, nj, SB0, nextF)) {
-                status = kStatusCapacity;
+            derive(w, A, tb, SB0, nextF);
+            pdirty = true;
+            if (Kadm < W) {
+                // window entry Kadm is the new head, and it does not fit at step t
+                h = w.win[Kadm];
+                hvalid = true;
                 break;
             }
             hvalid = false;
-            pdirty = true;
         }
         if (status != ST_OK) break;
         // ---- S6: process the batch
@@ -762,8 +820,9 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
             sumC += int64_t(c) * (int64_t(t) + 1);
             makespan = int64_t(t) + 1;
             ndone += c;
+            compact(w, A);
             tb = t + 1;
-            rebuild(w, A, tb, false, none, SB0, nextF);
+            derive(w, A, tb, SB0, nextF);
             pdirty = true;
             if (ndone >= n) break;
             ++t;
@@ -772,8 +831,7 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
             // next_a, (A_min) no overflow before tau_ov, and the head does not fit before tau_fit
             int64_t tau = nextF;
             if (ap < n) tau = min(tau, int64_t(next_a));
-            if (POL == P_AMIN && A > 0)
-                tau = min(tau, int64_t(tb) + floor_div(M - SB0, A) + 1);
+            if (POL == P_AMIN && A > 0) tau = min(tau, int64_t(tb) + floor_div(M - SB0, A) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
             if (tau > int64_t(t) + 1 && hvalid && A > 0)
                 tau = min(tau, first_fit_step(w, A, tb, SB0, M, t, h.s, h.key, tau));
@@ -802,14 +860,15 @@ __device__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     __syncwarp();
 }
 
-template <int POL>
+template <int POL, bool SMEM>
 __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
     const int wib = threadIdx.x >> 5;
     const int64_t slot = int64_t(blockIdx.x) * (blockDim.x >> 5) + wib;
-    unsigned char *base = P.use_smem ? smem_raw + size_t(wib) * ws_bytes_impl(P.ca, P.dcap)
-                                     : P.gws + slot * P.gws_stride;
+    unsigned char *base;
+    if (SMEM) base = smem_raw + size_t(wib) * ws_bytes_impl(P.ca, P.dcap);
+    else base = P.gws + slot * P.gws_stride;
     Ws w = carve_ws(base, P.ca, P.dcap);
     w.mb0 = P.mainbuf + slot * 2 * P.main_cap;
     w.mb1 = w.mb0 + P.main_cap;
@@ -823,24 +882,38 @@ __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
     }
 }
 
+template <int POL>
+const void *run_fn(bool smem) {
+    return smem ? (const void *)k_run<POL, true> : (const void *)k_run<POL, false>;
+}
+
 }  // namespace
 
 size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
-    const void *fn = policy == P_AMAX ? (const void *)k_run<P_AMAX>
-                   : policy == P_AMIN ? (const void *)k_run<P_AMIN>
-                                      : (const void *)k_run<P_HSF>;
+    const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true) : policy == P_AMIN ? run_fn<P_AMIN>(true)
+                                                                                : run_fn<P_HSF>(true);
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
 }
 
 cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
                        cudaStream_t st) {
     const dim3 grid(blocks), block(32 * warps_per_block);
+    const bool sm = p.use_smem != 0;
     switch (policy) {
-        case P_AMAX: k_run<P_AMAX><<<grid, block, smem_bytes, st>>>(p); break;
-        case P_AMIN: k_run<P_AMIN><<<grid, block, smem_bytes, st>>>(p); break;
-        default: k_run<P_HSF><<<grid, block, smem_bytes, st>>>(p); break;
+        case P_AMAX:
+            if (sm) k_run<P_AMAX, true><<<grid, block, smem_bytes, st>>>(p);
+            else k_run<P_AMAX, false><<<grid, block, smem_bytes, st>>>(p);
+            break;
+        case P_AMIN:
+            if (sm) k_run<P_AMIN, true><<<grid, block, smem_bytes, st>>>(p);
+            else k_run<P_AMIN, false><<<grid, block, smem_bytes, st>>>(p);
+            break;
+        default:
+            if (sm) k_run<P_HSF, true><<<grid, block, smem_bytes, st>>>(p);
+            else k_run<P_HSF, false><<<grid, block, smem_bytes, st>>>(p);
+            break;
     }
     return cudaGetLastError();
 }
