@@ -99,9 +99,11 @@ int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out);
  *   upper_u    u_i: predicted upper bound, o_i <= u_i.
  *   true_o     o_i >= 1: true output length (hidden from A_max and A_min; used by H-SF and by the
  *              simulation itself to know when a job finishes).
- *   device_ptrs 0: the arrays are host memory; 1: device memory on the current device.
- * The library copies the data into device buffers it owns; the caller may free or reuse its
- * arrays as soon as the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
+ *   device_ptrs 0: the arrays are host memory; 1: device memory on the current device, already
+ *               written (the call does not order itself after the caller's streams).
+ * The library copies the data into device buffers it owns (on a stream of its own, so the call
+ * does not wait for other work on the device); the caller may free or reuse its arrays as soon as
+ * the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
  * the call: they are reported in that instance's sim_result.status by sim_run.
  * Returns SIM_OK, SIM_E_INVAL (n_per_instance < 0, null pointer), SIM_E_NOMEM or SIM_E_CUDA.
  */

@@ -56,7 +56,11 @@ def build(force: bool = False, verbose: bool = False, extra: list[str] | None = 
         if verbose and out:
             print(out.decode(errors="replace"), file=sys.stderr)
     tmp = LIB.with_suffix(f".so.{os.getpid()}")
-    cmd = [cc, *ARCH, "-shared", "-o", str(tmp), *map(str, objs), "-cudart", "static"]
+    # the shared CUDA runtime: the library then sees the same current device and streams as the
+    # caller's runtime (e.g. torch.cuda.set_device in each rank / thread)
+    cudalib = str(Path(cc).parent.parent / "lib64")
+    cmd = [cc, *ARCH, "-shared", "-o", str(tmp), *map(str, objs), "-cudart", "shared",
+           "-Xlinker", f"-rpath,{cudalib}"]
     r = subprocess.run(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout.decode(errors='replace')}")

@@ -53,6 +53,7 @@ struct sim_ctx {
     QEnt *d_main = nullptr;
     size_t main_bytes = 0;
     double *d_cr = nullptr;
+    cudaStream_t load_stream = nullptr;  // non-blocking stream of sim_load (independent of other threads' work)
     int64_t launches = 0;
     std::vector<DevResult> h_res;
     std::string err;
@@ -200,14 +201,17 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
             return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_load: device allocation failed")
                                                   : cuda_fail(c, e, "cudaMalloc");
     }
+    if (!c->load_stream && (e = cudaStreamCreateWithFlags(&c->load_stream, cudaStreamNonBlocking)) != cudaSuccess)
+        return cuda_fail(c, e, "sim_load: stream creation");
+    const cudaStream_t ls = c->load_stream;
     const cudaMemcpyKind kind = device_ptrs ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
     const int32_t *src[5] = {a, s, l, u, o};
     for (int k = 0; k < 5; ++k) {
         if (nt == 0) break;
-        e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t), kind, 0);
+        e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t), kind, ls);
         if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the input arrays");
     }
-    e = cudaMemcpyAsync(c->d_off, offsets, size_t(c->n_inst + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, 0);
+    e = cudaMemcpyAsync(c->d_off, offsets, size_t(c->n_inst + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, ls);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the offsets");
     simgb::StageParams sp;
     sp.policy = c->policy;
@@ -223,10 +227,10 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
     sp.rec = c->d_rec;
     sp.rec_a = c->d_rec_a;
     sp.info = c->d_info;
-    e = simgb::launch_stage(sp, 0);
+    e = simgb::launch_stage(sp, ls);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: staging kernel launch");
     if (c->n_inst > 0) ++c->launches;
-    e = cudaStreamSynchronize(0);
+    e = cudaStreamSynchronize(ls);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: staging kernel");
     c->n_total = nt;
     c->n_max = int32_t(n_max);
@@ -433,6 +437,7 @@ void sim_destroy(sim_ctx *c) {
     dfree(c->d_gws);
     dfree(c->d_main);
     dfree(c->d_cr);
+    if (c->load_stream) cudaStreamDestroy(c->load_stream);
     delete c;
 }
 

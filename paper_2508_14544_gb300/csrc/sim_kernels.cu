@@ -469,15 +469,83 @@ __device__ __forceinline__ void compact(const Ws &w, int &A) {
     A = wpos;
 }
 
+// Remove the entries marked dead (F < 0) and recompute the derived arrays, in one pass when the
+// set fits one chunk (positions, suffix sums and prefix maxima of the compacted order are known
+// from the live counts before anything is stored).
+__device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int &SB0, int &nextF) {
+    if (A > kChunk) {
+        compact(w, A);
+        derive(w, A, tb, SB0, nextF);
+        return;
+    }
+    const int lane = lane_id();
+    const int base = 4 * lane;
+    const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
+    const int4 p4 = ld4(w.P, base), i4 = ld4(w.I, base), k4 = ld4(w.K, base);
+    const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
+    const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
+    const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+    bool lv[4];
+    int lc = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        lv[j] = (base + j < A) && ff[j] >= 0;
+        lc += lv[j] ? 1 : 0;
+    }
+    int L;
+    const int off = excl_scan_add(lc, L);
+    int sfx[4];
+    int acc = 0;
+#pragma unroll
+    for (int j = 3; j >= 0; --j) {
+        acc += lv[j] ? bb[j] + tb : 0;
+        sfx[j] = acc;
+    }
+    int tot;
+    const int after = excl_suffix_add(acc, tot);
+    int q = off, mx = INT_MIN, fmin = INT_MAX;
+    int qp[4], mm[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        qp[j] = q;
+        if (lv[j]) {
+            const int64_t e = int64_t(ee[j]) - tb;
+            mx = max(mx, sat32(int64_t(sfx[j] + after) + int64_t(L - q) * e + e));
+            fmin = min(fmin, ff[j]);
+            ++q;
+        }
+        mm[j] = mx;
+    }
+    const int before = excl_scan_max(mx);
+    nextF = __reduce_min_sync(FULL, fmin);
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (lv[j]) {
+            store_job(w, qp[j], ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
+            w.SB[qp[j]] = sfx[j] + after;
+            w.PM[qp[j] + 1] = max(before, mm[j]);
+        }
+    }
+    if (lane == 0) {
+        w.SB[L] = 0;
+        w.PM[0] = INT_MIN;
+    }
+    A = L;
+    SB0 = tot;
+    __syncwarp();
+}
+
 // Insert the K window entries admitted at step t (lane m < K holds entry m, ascending E) into the
-// compact active set, keeping E ascending (new entries after equal old ones).  Entries only move
-// right, so chunks are processed from the back.  Returns false if the capacity is exceeded.
+// compact active set, keeping E ascending (new entries after equal old ones): with
+// cnt_m = #{old E <= E_m}, new entry m goes to m + cnt_m and old entry p moves right by
+// #{m : cnt_m <= p}.  Entries only move right, so chunks are processed from the back.
+// Returns false if the capacity is exceeded.
 __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t, const QEnt &mine) {
     const int lane = lane_id();
     if (A + K > w.ca) return false;
     const int ne = t + mine.key - 1;
-    // destination of new entry m: m + #{old E <= E_m}
-    const int posm = (lane < K) ? lane + lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; }) : 0;
+    const int cnt = (lane < K) ? lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; }) : INT_MAX;
     const int last = ((A - 1) / kChunk) * kChunk;
     for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
         const int base = cb + 4 * lane;
@@ -486,12 +554,11 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
         const int ee[4] = {e4.x, e4.y, e4.z, e4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
         const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
         const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-        int sh[4];
+        int sh[4] = {0, 0, 0, 0};
+        for (int m = 0; m < K; ++m) {
+            const int c = __shfl_sync(FULL, cnt, m);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            // #{new m < K: E_m < E_j},  E_m = t + key_m - 1 ascending in m
-            const int lim = ee[j] - t + 1;  // E_m < E_j  <=>  key_m < lim
-            sh[j] = (base + j < A) ? lane_prefix_count(K, [&](int m) { return w.wkey[m] < lim; }) : 0;
+            for (int j = 0; j < 4; ++j) sh[j] += (base + j >= c) ? 1 : 0;
         }
         __syncwarp();
 #pragma unroll
@@ -499,7 +566,7 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
             if (base + j < A) store_job(w, base + j + sh[j], ee[j], ff[j], bb[j], pp[j], ii[j], kk[j]);
         __syncwarp();
     }
-    if (lane < K) store_job(w, posm, ne, t + mine.o - 1, mine.s - t + 1, t, mine.idx, mine.key);
+    if (lane < K) store_job(w, lane + cnt, ne, t + mine.o - 1, mine.s - t + 1, t, mine.idx, mine.key);
     __syncwarp();
     A += K;
     return true;
@@ -714,22 +781,21 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                     }
                     const int pos = __shfl_sync(FULL, bp, __ffs(ball) - 1);
                     const int b = w.B[pos], p = w.P[pos], f = w.F[pos], k = w.K[pos], id = w.I[pos];
-                    __syncwarp();
-                    if (lane == 0) w.F[pos] = -1;
-                    __syncwarp();
                     QEnt e;
                     e.key = max(k, t - p);  // refined lower bound: max(estimate, tokens generated)
                     e.idx = id;
                     e.s = b + p - 1;
                     e.o = f - p + 1;
+                    __syncwarp();
+                    if (lane == 0) w.F[pos] = -1;
+                    __syncwarp();
                     need -= int64_t(b) + t;
                     ++nev;
                     delta_insert(w, q, e);
                 }
                 if (status != ST_OK) break;
-                compact(w, A);
                 tb = t;
-                derive(w, A, tb, SB0, nextF);
+                compact_derive(w, A, tb, SB0, nextF);
                 hvalid = false;
                 pdirty = true;
             }
@@ -820,9 +886,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             sumC += int64_t(c) * (int64_t(t) + 1);
             makespan = int64_t(t) + 1;
             ndone += c;
-            compact(w, A);
             tb = t + 1;
-            derive(w, A, tb, SB0, nextF);
+            compact_derive(w, A, tb, SB0, nextF);
             pdirty = true;
             if (ndone >= n) break;
             ++t;
