@@ -49,6 +49,7 @@ enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
 enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
 constexpr int kChunk = 128;  // active-set entries per warp pass (4 per lane)
 constexpr int kWin = 32;     // admission window (one candidate per lane)
+constexpr int kMc = 64;      // cached entries of the main queue (two per lane)
 constexpr int64_t kBig = int64_t(1) << 60;
 
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
@@ -147,7 +148,7 @@ struct Ws {
     int32_t *SB, *PM;                // ca + 4
     QEnt *dq;                        // delta queue, dcap entries, sorted DESCENDING (head = dq[dn-1])
     QEnt *win;                       // admission window, kWin entries in (key, idx) order
-    QEnt *mc;                        // cached head of the main queue, kWin entries
+    QEnt *mc;                        // cached head of the main queue, kMc entries
     int32_t *cnt;                    // dcap + 4 (merge histogram)
     int32_t *wkey, *wcs, *wsrc;      // window keys, prefix sums CS[0..kWin], sources (0 main, 1 delta)
     QEnt *mb0, *mb1;                 // global ping-pong main-queue buffers
@@ -157,7 +158,7 @@ struct Ws {
 __host__ __device__ inline size_t ws_bytes_impl(int ca, int dcap) {
     size_t b = size_t(6) * ca * sizeof(int32_t) + size_t(2) * (ca + 4) * sizeof(int32_t);
     b = (b + 15) & ~size_t(15);
-    b += size_t(dcap + 2 * kWin) * sizeof(QEnt);
+    b += size_t(dcap + kWin + kMc) * sizeof(QEnt);
     b += size_t(dcap + 4) * sizeof(int32_t) + size_t(kWin + kWin + 4 + kWin) * sizeof(int32_t);
     return (b + 15) & ~size_t(15);
 }
@@ -178,7 +179,7 @@ __device__ __forceinline__ Ws carve_ws(unsigned char *base, int ca, int dcap) {
     w.dq = reinterpret_cast<QEnt *>(base + off);
     w.win = w.dq + dcap;
     w.mc = w.win + kWin;
-    w.cnt = reinterpret_cast<int32_t *>(w.mc + kWin);
+    w.cnt = reinterpret_cast<int32_t *>(w.mc + kMc);
     w.wkey = w.cnt + dcap + 4;
     w.wcs = w.wkey + kWin;
     w.wsrc = w.wcs + kWin + 4;
@@ -200,16 +201,22 @@ struct Queue {
     int mh, me;      // head / end
     int mbuf;        // -1: mq is read-only staged data; 0/1: ping-pong buffer in use
     int dn;          // delta size
-    int mcb;         // main cache base: w.mc[i] = mq[mcb + i]; -1 invalid
+    int mcb;         // main cache base: w.mc[i] = mq[mcb + i] for i < kMc; -1 invalid
 };
 
 __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.me && q.dn == 0; }
 
-// Make w.mc hold mq[mh .. mh + kWin).
+// Make w.mc cover mq[mh .. mh + kWin): keep the cached run while the head is within its first
+// kMc - kWin entries, otherwise reload kMc entries from the head.
 __device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
-    if (q.mcb == q.mh) return;
-    const int i = q.mh + lane_id();
-    if (i < q.me) w.mc[lane_id()] = q.mq[i];
+    if (q.mcb >= 0 && q.mh >= q.mcb && q.mh - q.mcb <= kMc - kWin) return;
+    const int lane = lane_id();
+    const int i0 = q.mh + lane, i1 = q.mh + 32 + lane;
+    QEnt a, b;
+    if (i0 < q.me) a = q.mq[i0];
+    if (i1 < q.me) b = q.mq[i1];
+    if (i0 < q.me) w.mc[lane] = a;
+    if (i1 < q.me) w.mc[32 + lane] = b;
     __syncwarp();
     q.mcb = q.mh;
 }
@@ -294,10 +301,7 @@ __device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q) {
     const bool have_m = q.mh < q.me;
     QEnt hm;
     if (have_m) {
-        if (q.mcb < 0 || q.mh < q.mcb || q.mh >= q.mcb + kWin) {
-            q.mcb = -1;
-            main_cache_at_head(w, q);
-        }
+        main_cache_at_head(w, q);
         hm = w.mc[q.mh - q.mcb];
     }
     if (q.dn > 0) {
@@ -344,8 +348,9 @@ __device__ __forceinline__ int build_window(const Ws &w, Queue &q) {
     const int nm = min(kWin, max(nmain, 0));
     const int dn = q.dn;
     const int nd = min(kWin, dn);
+    const int mo = q.mh - q.mcb;  // offset of the head in the cache
     if (lane < nm) {
-        const QEnt x = w.mc[lane];
+        const QEnt x = w.mc[mo + lane];
         const int r = lane_prefix_count(dn, [&](int m) { return qless(w.dq[dn - 1 - m], x); });
         const int pos = lane + r;
         if (pos < kWin) {
@@ -355,7 +360,7 @@ __device__ __forceinline__ int build_window(const Ws &w, Queue &q) {
     }
     if (lane < nd) {
         const QEnt y = w.dq[dn - 1 - lane];
-        const int c = lane_prefix_count(nm, [&](int m) { return qless(w.mc[m], y); });
+        const int c = lane_prefix_count(nm, [&](int m) { return qless(w.mc[mo + m], y); });
         const int pos = lane + c;
         if (pos < kWin) {
             w.win[pos] = y;
@@ -572,10 +577,11 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
     return true;
 }
 
-// Largest admissible prefix of the window at step t (see the file comment).  Lane m holds window
-// entry m (m < W); the active set is compact with derived arrays for time base tb.
-__device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int W,
-                                                 const QEnt &mine) {
+// Largest admissible prefix of the window at step t (see the file comment), for any active-set
+// size: per point a binary search for the first failing prefix length.  Lane m holds window entry
+// m (m < W); the active set is compact with derived arrays for time base tb.
+__device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int tb, int SB0, int64_t M, int t,
+                                                        int W, const QEnt &mine) {
     const int lane = lane_id();
     // prefix sums CS[k] = sum_{m<k} (s_m + 1)
     int tot;
@@ -634,6 +640,56 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     }
     phi = __reduce_min_sync(FULL, phi);
     return min(max(phi - 1, 0), W);
+}
+
+// Largest admissible prefix of the window at step t when the active set fits one chunk: every
+// point keeps its projected memory in a register and the window entries are added one at a time
+// (candidate k-1 adds s + 1 + (x - t) at every point x it reaches: the coming step x = t, the
+// active endpoints E_j with key > E_j - t, and the endpoints of window entries 0..k-1); the first
+// k at which any point exceeds M ends the prefix.  Falls back to the binary-search form otherwise.
+__device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int W,
+                                                 const QEnt &mine) {
+    if (A > kChunk) return admissible_prefix_search(w, A, tb, SB0, M, t, W, mine);
+    const int lane = lane_id();
+    const int Mi = int(M);
+    // active endpoints at or after t: V(E_j) and d_j = E_j - t
+    const int base = 4 * lane;
+    const int4 e4 = ld4(w.E, base), s4 = ld4(w.SB, base);
+    const int ee[4] = {e4.x, e4.y, e4.z, e4.w};
+    const int ss[4] = {s4.x, s4.y, s4.z, s4.w};
+    int va[4], da[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const bool ok = base + j < A && ee[j] >= t;
+        da[j] = ok ? ee[j] - t : INT_MAX;
+        va[j] = ok ? sat32(int64_t(ss[j]) + int64_t(A - base - j) * (int64_t(ee[j]) - tb)) : INT_MIN;
+    }
+    // this lane's window entry: V(y) of the active set at its last step y = t + key - 1
+    const int dm = mine.key - 1;
+    int vc = INT_MIN;
+    int av = 0;
+    if (lane < W) {
+        const int64_t y = int64_t(t) + dm;
+        const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
+        av = sat32(int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb));
+    }
+    int64_t need = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
+    for (int k = 1; k <= W; ++k) {
+        const int sk = __shfl_sync(FULL, mine.s, k - 1) + 1;
+        const int kk = __shfl_sync(FULL, mine.key, k - 1);
+        need += sk;
+        bool fail = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (kk > da[j]) va[j] += sk + da[j];
+            fail = fail || va[j] > Mi;
+        }
+        if (lane == k - 1) vc = av + sk + dm;
+        else if (lane < k - 1) vc += sk + dm;
+        fail = fail || vc > Mi;
+        if (__ballot_sync(FULL, fail) != 0 || need > M) return k - 1;
+    }
+    return W;
 }
 
 // First step tau in (t, tau_lim) at which the head candidate (prompt s, estimate L) fits, with the

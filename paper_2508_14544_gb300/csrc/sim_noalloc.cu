@@ -47,7 +47,7 @@ constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 constexpr size_t ws_bytes_max() {
     size_t b = size_t(6) * kNaMaxPerInstance * 4 + size_t(2) * (kNaMaxPerInstance + 4) * 4;
     b = (b + 15) & ~size_t(15);
-    b += size_t(kNaDeltaCap + 64) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 4 + 100) * 4;
+    b += size_t(kNaDeltaCap + 96) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 4 + 100) * 4;
     return (b + 15) & ~size_t(15);
 }
 
