@@ -72,10 +72,13 @@ enum {
     SIM_OPT_RECORD_COMPLETIONS = 2, /* 0/1: keep each request's completion step for
                                        sim_get_completions (default 0). */
     SIM_OPT_WARPS_PER_BLOCK = 3,    /* 1..8: simulation warps per thread block (default 4). */
-    SIM_OPT_SMEM_ACTIVE_CAP = 4     /* 128..4096, multiple of 128: active-set slots kept in shared
+    SIM_OPT_SMEM_ACTIVE_CAP = 4,    /* 128..4096, multiple of 128: active-set slots kept in shared
                                        memory per instance (default 512).  Instances that need more
                                        are re-run automatically with the active set in global
                                        memory; results are identical. */
+    SIM_OPT_WARPS_PER_SM = 5        /* 0..64: at most this many simulation warps resident per SM
+                                       (0, the default: as many as shared memory allows).  Results
+                                       do not depend on it. */
 };
 
 /*

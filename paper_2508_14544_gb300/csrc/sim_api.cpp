@@ -28,6 +28,7 @@ struct sim_ctx {
     int64_t step_cap = 0;
     int record_completions = 0;
     int wpb = 4;
+    int warps_per_sm = 0;
     int smem_ca = 512;
     int dcap = 256;
     // state
@@ -148,6 +149,10 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
         case SIM_OPT_WARPS_PER_BLOCK:
             if (value < 1 || value > 8) return fail(c, SIM_E_INVAL, "WARPS_PER_BLOCK must be in [1, 8]");
             c->wpb = int(value);
+            return SIM_OK;
+        case SIM_OPT_WARPS_PER_SM:
+            if (value < 0 || value > 64) return fail(c, SIM_E_INVAL, "WARPS_PER_SM must be in [0, 64]");
+            c->warps_per_sm = int(value);
             return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
             if (value < 128 || value > 4096 || value % 128)
@@ -274,6 +279,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     } else {
         per_sm = std::max(1, 16 / wpb);
     }
+    if (c->warps_per_sm > 0) per_sm = std::max(1, std::min(per_sm, c->warps_per_sm / wpb));
     int64_t blocks = int64_t(n_sm) * per_sm;
     blocks = std::min<int64_t>(blocks, (n_work + wpb - 1) / wpb);
     blocks = std::max<int64_t>(blocks, 1);

@@ -63,9 +63,13 @@ __device__ __forceinline__ int sat32(int64_t v) {
     return int(v > hi ? hi : (v < -hi ? -hi : v));
 }
 
-__device__ __forceinline__ int64_t floor_div(int64_t a, int64_t b) {  // b > 0
-    int64_t q = a / b;
-    if ((a % b != 0) && (a < 0)) --q;
+// floor(a / b) for b > 0 in 32-bit arithmetic.  The numerators here are M minus memory sums that
+// are >= 0, so they are <= M <= 2^26; a numerator below -2^30 is raised to -2^30, which keeps the
+// quotient negative enough for every use (each one only asks whether a step lies before t).
+__device__ __forceinline__ int floor_div32(int64_t a, int b) {
+    const int ai = int(max(min(a, int64_t(INT_MAX)), -(int64_t(1) << 30)));
+    int q = ai / b;
+    if ((ai % b != 0) && (ai < 0)) --q;
     return q;
 }
 
@@ -147,10 +151,9 @@ struct Ws {
     int32_t *E, *F, *B, *P, *I, *K;  // active set, capacity ca (multiple of kChunk), 16-byte aligned
     int32_t *SB, *PM;                // ca + 4
     QEnt *dq;                        // delta queue, dcap entries, sorted DESCENDING (head = dq[dn-1])
-    QEnt *win;                       // admission window, kWin entries in (key, idx) order
     QEnt *mc;                        // cached head of the main queue, kMc entries
     int32_t *cnt;                    // dcap + 4 (merge histogram)
-    int32_t *wkey, *wcs, *wsrc;      // window keys, prefix sums CS[0..kWin], sources (0 main, 1 delta)
+    int32_t *wkey, *wcs;             // window keys and prefix sums CS[0..kWin] (wide-set prefix search)
     QEnt *mb0, *mb1;                 // global ping-pong main-queue buffers
     int32_t ca, dcap;
 };
@@ -158,8 +161,8 @@ struct Ws {
 __host__ __device__ inline size_t ws_bytes_impl(int ca, int dcap) {
     size_t b = size_t(6) * ca * sizeof(int32_t) + size_t(2) * (ca + 4) * sizeof(int32_t);
     b = (b + 15) & ~size_t(15);
-    b += size_t(dcap + kWin + kMc) * sizeof(QEnt);
-    b += size_t(dcap + 4) * sizeof(int32_t) + size_t(kWin + kWin + 4 + kWin) * sizeof(int32_t);
+    b += size_t(dcap + kMc) * sizeof(QEnt);
+    b += size_t(dcap + 4) * sizeof(int32_t) + size_t(kWin + kWin + 4) * sizeof(int32_t);
     return (b + 15) & ~size_t(15);
 }
 
@@ -177,12 +180,10 @@ __device__ __forceinline__ Ws carve_ws(unsigned char *base, int ca, int dcap) {
     size_t off = size_t(reinterpret_cast<unsigned char *>(p) - base);
     off = (off + 15) & ~size_t(15);
     w.dq = reinterpret_cast<QEnt *>(base + off);
-    w.win = w.dq + dcap;
-    w.mc = w.win + kWin;
+    w.mc = w.dq + dcap;
     w.cnt = reinterpret_cast<int32_t *>(w.mc + kMc);
     w.wkey = w.cnt + dcap + 4;
     w.wcs = w.wkey + kWin;
-    w.wsrc = w.wcs + kWin + 4;
     w.ca = ca;
     w.dcap = dcap;
     return w;
@@ -221,48 +222,52 @@ __device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
     q.mcb = q.mh;
 }
 
-// Merge the delta into the main array (into the other ping-pong buffer).
-__device__ __forceinline__ void merge_delta(const Ws &w, Queue &q) {
+// Merge the delta into the main array (into the other ping-pong buffer).  Rare (a full delta, or
+// a long arrival run), so it is kept out of line: the simulation loop stays small enough for the
+// instruction cache when two warps share a scheduler.  Takes the few workspace pointers it needs
+// by value and the queue by pointer.
+__device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0, QEnt *mb1, Queue *qp) {
     const int lane = lane_id();
+    Queue q = *qp;
     const int dn = q.dn;
     const int nx = q.me - q.mh;
-    QEnt *out = (q.mbuf == 0) ? w.mb1 : w.mb0;
+    QEnt *out = (q.mbuf == 0) ? mb1 : mb0;
     const QEnt *X = q.mq + q.mh;
-    for (int j = lane; j <= dn; j += 32) w.cnt[j] = 0;
+    for (int j = lane; j <= dn; j += 32) cnt[j] = 0;
     __syncwarp();
     const int c = (nx + 31) >> 5;
     const int s0 = lane * c;
     const int s1 = min(s0 + c, nx);
     if (s0 < s1) {
         const QEnt x0 = X[s0];
-        int r = lane_prefix_count(dn, [&](int m) { return qless(w.dq[dn - 1 - m], x0); });
+        int r = lane_prefix_count(dn, [&](int m) { return qless(dq[dn - 1 - m], x0); });
         int run_r = r, run_len = 0;
         for (int i = s0; i < s1; ++i) {
             const QEnt x = X[i];
-            while (r < dn && qless(w.dq[dn - 1 - r], x)) ++r;
+            while (r < dn && qless(dq[dn - 1 - r], x)) ++r;
             out[i + r] = x;
             if (r != run_r) {
-                if (run_len) atomicAdd(&w.cnt[run_r], run_len);
+                if (run_len) atomicAdd(&cnt[run_r], run_len);
                 run_r = r;
                 run_len = 0;
             }
             ++run_len;
         }
-        if (run_len) atomicAdd(&w.cnt[run_r], run_len);
+        if (run_len) atomicAdd(&cnt[run_r], run_len);
     }
     __syncwarp();
     // delta element j (ascending) goes to j + #{main entries smaller} = j + sum_{r <= j} cnt[r]
     int carry = 0;
     for (int c0 = 0; c0 < dn; c0 += 32) {
         const int j = c0 + lane;
-        int v = (j < dn) ? w.cnt[j] : 0;
+        int v = (j < dn) ? cnt[j] : 0;
 #pragma unroll
         for (int d = 1; d < 32; d <<= 1) {
             const int y = __shfl_up_sync(FULL, v, d);
             if (lane >= d) v += y;
         }
         v += carry;
-        if (j < dn) out[j + v] = w.dq[dn - 1 - j];
+        if (j < dn) out[j + v] = dq[dn - 1 - j];
         carry = __shfl_sync(FULL, v, 31);
     }
     __syncwarp();
@@ -273,6 +278,13 @@ __device__ __forceinline__ void merge_delta(const Ws &w, Queue &q) {
     q.me = nx + dn;
     q.dn = 0;
     q.mcb = -1;
+    *qp = q;
+}
+
+__device__ __forceinline__ void merge_delta(const Ws &w, Queue &q) {
+    Queue qq = q;
+    merge_delta(w.cnt, w.dq, w.mb0, w.mb1, &qq);
+    q = qq;
 }
 
 // Insert one entry into the delta (merging the delta into main first if it is full).
@@ -340,35 +352,32 @@ __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *ru
     }
 }
 
-// First kWin entries of R_t in (key, idx) order into w.win / w.wsrc; returns how many.
-__device__ __forceinline__ int build_window(const Ws &w, Queue &q) {
+// First kWin entries of R_t in (key, idx) order, by a merge path over the cached head of the main
+// array (ascending) and the delta (descending): lane m finds how many of the m smallest entries
+// come from the main array and returns entry m in `mine` (src 0 main, 1 delta).  Returns how many.
+__device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, int &msrc) {
     const int lane = lane_id();
-    const int nmain = q.me - q.mh;
+    const int nmain = max(q.me - q.mh, 0);
     if (nmain > 0) main_cache_at_head(w, q);
-    const int nm = min(kWin, max(nmain, 0));
+    const int na = min(kWin, nmain);
     const int dn = q.dn;
-    const int nd = min(kWin, dn);
-    const int mo = q.mh - q.mcb;  // offset of the head in the cache
-    if (lane < nm) {
-        const QEnt x = w.mc[mo + lane];
-        const int r = lane_prefix_count(dn, [&](int m) { return qless(w.dq[dn - 1 - m], x); });
-        const int pos = lane + r;
-        if (pos < kWin) {
-            w.win[pos] = x;
-            w.wsrc[pos] = 0;
-        }
+    const int nb = min(kWin, dn);
+    const QEnt *A = w.mc + (q.mh - q.mcb);  // A[i], ascending
+    const QEnt *Bd = w.dq + (dn - 1);       // B[j] = Bd[-j], ascending
+    int lo = max(0, lane - nb), hi = min(lane, na);
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (qless(A[mid], Bd[-(lane - 1 - mid)])) lo = mid + 1; else hi = mid;
     }
-    if (lane < nd) {
-        const QEnt y = w.dq[dn - 1 - lane];
-        const int c = lane_prefix_count(nm, [&](int m) { return qless(w.mc[mo + m], y); });
-        const int pos = lane + c;
-        if (pos < kWin) {
-            w.win[pos] = y;
-            w.wsrc[pos] = 1;
-        }
+    const int j = lane - lo;
+    const int W = min(kWin, na + nb);
+    msrc = 0;
+    if (lane < W) {
+        const bool take_a = j >= nb || (lo < na && qless(A[lo], Bd[-j]));
+        mine = take_a ? A[lo] : Bd[-j];
+        msrc = take_a ? 0 : 1;
     }
-    __syncwarp();
-    return min(kWin, max(nmain, 0) + dn);
+    return W;
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -674,20 +683,35 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
         av = sat32(int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb));
     }
     int64_t need = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
-    for (int k = 1; k <= W; ++k) {
-        const int sk = __shfl_sync(FULL, mine.s, k - 1) + 1;
-        const int kk = __shfl_sync(FULL, mine.key, k - 1);
-        need += sk;
-        bool fail = false;
+    // two candidates per round: the state after both is used only if neither fails
+    for (int k = 1; k <= W; k += 2) {
+        const bool two = k < W;
+        const int s1 = __shfl_sync(FULL, mine.s, k - 1) + 1;
+        const int k1 = __shfl_sync(FULL, mine.key, k - 1);
+        const int s2 = __shfl_sync(FULL, mine.s, k) + 1;
+        const int k2 = __shfl_sync(FULL, mine.key, k);
+        const int64_t need1 = need + s1;
+        const int64_t need2 = need1 + s2;
+        bool f1 = false, f2 = false;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            if (kk > da[j]) va[j] += sk + da[j];
-            fail = fail || va[j] > Mi;
+            if (k1 > da[j]) va[j] += s1 + da[j];
+            f1 = f1 || va[j] > Mi;
+            if (k2 > da[j]) va[j] += s2 + da[j];
+            f2 = f2 || va[j] > Mi;
         }
-        if (lane == k - 1) vc = av + sk + dm;
-        else if (lane < k - 1) vc += sk + dm;
-        fail = fail || vc > Mi;
-        if (__ballot_sync(FULL, fail) != 0 || need > M) return k - 1;
+        if (lane == k - 1) vc = av + s1 + dm;
+        else if (lane < k - 1) vc += s1 + dm;
+        f1 = f1 || vc > Mi;
+        if (lane == k) vc = av + s2 + dm;
+        else if (lane < k) vc += s2 + dm;
+        f2 = f2 || vc > Mi;
+        const unsigned b1 = __ballot_sync(FULL, f1);
+        const unsigned b2 = __ballot_sync(FULL, f2);
+        if (b1 != 0 || need1 > M) return k - 1;
+        if (!two) break;
+        if (b2 != 0 || need2 > M) return k;
+        need = need2;
     }
     return W;
 }
@@ -703,7 +727,7 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
     const int lane = lane_id();
     const int64_t y0 = int64_t(t) + L - 1;
     const int64_t ylim = tau_lim - 1 + L - 1;
-    const int64_t tau1 = tb + floor_div(M - s - 1 - SB0, A);  // (1)
+    const int64_t tau1 = tb + floor_div32(M - s - 1 - SB0, A);  // (1)
     const int64_t yup = min(ylim, tau1 + L - 1);
     if (yup <= y0) return kBig;
     const int64_t C2 = M - s - L - tb;
@@ -713,7 +737,7 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
         const int64_t prev = (j == 0) ? -kBig : int64_t(w.E[j - 1]);
         const int64_t cur = (j == A) ? kBig : int64_t(w.E[j]);
         if (cur <= y0 || prev >= yup) continue;
-        const int64_t y3 = (A - j > 0) ? tb + floor_div(C3 - w.SB[j], A - j) : kBig;
+        const int64_t y3 = (A - j > 0) ? tb + floor_div32(C3 - w.SB[j], A - j) : kBig;
         const int64_t up = min(yup, y3);
         const int64_t lo = max(prev + 1, y0 + 1);
         const int64_t cand = max(lo, int64_t(w.PM[j]) - C2);
@@ -776,7 +800,18 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
     int64_t y_prev = 0;
     int hi = 0, lb = 0;
 
+    bool pend_compact = false;
+    int tb_next = 0;
     for (;;) {
+        if (pend_compact) {
+            // jobs marked dead (cancelled or completed) leave the active set.  Both kinds of
+            // removal share this one site: the loop body stays small, which matters when two
+            // warps at different points of it share a scheduler's instruction cache.
+            tb = tb_next;
+            compact_derive(w, A, tb, SB0, nextF);
+            pend_compact = false;
+            pdirty = true;
+        }
         if (steps >= cap) {
             status = ST_STEPCAP;
             break;
@@ -850,10 +885,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                     delta_insert(w, q, e);
                 }
                 if (status != ST_OK) break;
-                tb = t;
-                compact_derive(w, A, tb, SB0, nextF);
+                tb_next = t;
+                pend_compact = true;
                 hvalid = false;
-                pdirty = true;
+                continue;
             }
         }
         // ---- S4/S5: admit the largest feasible prefix of R_t
@@ -887,14 +922,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             }
             if (!fits) break;
             // the head fits: find the whole admissible prefix on the window
-            const int W = build_window(w, q);
             QEnt mine;
             mine.key = mine.idx = mine.s = mine.o = 0;
             int msrc = 0;
-            if (lane < W) {
-                mine = w.win[lane];
-                msrc = w.wsrc[lane];
-            }
+            const int W = build_window(w, q, mine, msrc);
             const int Kadm = admissible_prefix(w, A, tb, SB0, M, t, W, mine);
             if (Kadm <= 0) {
                 status = ST_STATE;  // the head test and the window disagree: internal error
@@ -912,7 +943,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             pdirty = true;
             if (Kadm < W) {
                 // window entry Kadm is the new head, and it does not fit at step t
-                h = w.win[Kadm];
+                h.key = __shfl_sync(FULL, mine.key, Kadm);
+                h.idx = __shfl_sync(FULL, mine.idx, Kadm);
+                h.s = __shfl_sync(FULL, mine.s, Kadm);
+                h.o = __shfl_sync(FULL, mine.o, Kadm);
                 hvalid = true;
                 break;
             }
@@ -942,17 +976,16 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             sumC += int64_t(c) * (int64_t(t) + 1);
             makespan = int64_t(t) + 1;
             ndone += c;
-            tb = t + 1;
-            compact_derive(w, A, tb, SB0, nextF);
-            pdirty = true;
             if (ndone >= n) break;
+            tb_next = t + 1;
+            pend_compact = true;
             ++t;
         } else {
             // steps t .. tau-1 change nothing: no completion before nextF, no arrival before
             // next_a, (A_min) no overflow before tau_ov, and the head does not fit before tau_fit
             int64_t tau = nextF;
             if (ap < n) tau = min(tau, int64_t(next_a));
-            if (POL == P_AMIN && A > 0) tau = min(tau, int64_t(tb) + floor_div(M - SB0, A) + 1);
+            if (POL == P_AMIN && A > 0) tau = min(tau, int64_t(tb) + floor_div32(M - SB0, A) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
             if (tau > int64_t(t) + 1 && hvalid && A > 0)
                 tau = min(tau, first_fit_step(w, A, tb, SB0, M, t, h.s, h.key, tau));

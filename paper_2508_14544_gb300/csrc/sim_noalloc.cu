@@ -41,13 +41,13 @@ constexpr int kNaDeltaCap = 256;
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Workspace bytes per warp for an active-set capacity of kNaMaxPerInstance (same formula as the
-// simulation kernel's carve: 6 x ca + 2 x (ca + 4) int32, 16-byte aligned, then the delta queue,
-// the admission window and the main-queue head cache, and the int32 scratch of the window and
-// the merge histogram).  A run-time check compares it with the kernel's own size.
+// simulation kernel's carve: 6 x ca + 2 x (ca + 4) int32, 16-byte aligned, then the delta queue
+// and the main-queue head cache, and the int32 scratch of the window and the merge histogram).
+// A run-time check compares it with the kernel's own size.
 constexpr size_t ws_bytes_max() {
     size_t b = size_t(6) * kNaMaxPerInstance * 4 + size_t(2) * (kNaMaxPerInstance + 4) * 4;
     b = (b + 15) & ~size_t(15);
-    b += size_t(kNaDeltaCap + 96) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 4 + 100) * 4;
+    b += size_t(kNaDeltaCap + 64) * sizeof(simgb::QEnt) + size_t(kNaDeltaCap + 4 + 68) * 4;
     return (b + 15) & ~size_t(15);
 }
 
