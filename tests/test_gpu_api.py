@@ -93,13 +93,27 @@ def test_host_and_device_loads_and_reruns_agree():
             assert np.array_equal(r1[f], r2[f]) and np.array_equal(r1[f], a[f])
 
 
-@pytest.mark.parametrize("wpb", [1, 2, 8])
-def test_launch_shapes_agree(wpb):
+@pytest.mark.parametrize("wpb,wps", [(1, 0), (2, 0), (8, 0), (4, 4)])
+def test_launch_shapes_agree(wpb, wps):
+    """Warps per block and resident warps per SM change only the schedule of instances on the
+    GPU, never a result."""
     from paper_2508_14544_gb300 import workloads as W
     w = W.make_workload("c2", range(5, 1024, 41))
     for pol in (0, 1, 2):
         a, _ = gpu_run(pol, w)
-        b, _ = gpu_run(pol, w, warps_per_block=wpb)
+        b, _ = gpu_run(pol, w, warps_per_block=wpb, warps_per_sm=wps)
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f])
+
+
+def test_more_instances_than_warps():
+    """One resident warp per SM (152 warps) for 342 instances: every warp simulates several
+    instances in turn, reusing its workspace, and the results do not change."""
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(0, 1024, 3))
+    for pol in (0, 1, 2):
+        a, _ = gpu_run(pol, w)
+        b, _ = gpu_run(pol, w, warps_per_block=1, warps_per_sm=1)
         for f in FIELDS:
             assert np.array_equal(a[f], b[f])
 
