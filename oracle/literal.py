@@ -1,4 +1,4 @@
-"""Literal CPU oracle of the batched schedulers (A_max, A_min, H-SF).
+"""Literal CPU oracle of the batched schedulers (A_max, A_min, H-SF, A_r, A_ell).
 
 TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import this module.  The CUDA path shares no code with it.
@@ -41,6 +41,22 @@ Readings of the text that this oracle fixes (each is also listed in the design n
   g_i <- 0, back to the waiting set, and eligible in the same step's admission ("unprocessed or
   restartable requests", Section 4).  Both the max and the same-step eligibility are switchable
   for sensitivity studies (``refine`` / ``same_step``).
+* A_r (Algorithm random, Appendix B).  The true lengths o, and a fixed random permutation given as
+  ``rank`` (rank[i] = position of request i; the draw is an input, not made here).  Admission is
+  the largest feasible prefix of the waiting set in (rank, index) order, as for the other
+  policies.
+* A_ell (Algorithm promote_l, Section 5 and Appendix).  The waiting set is a FIFO queue: a request
+  enters it at its arrival step, and a promoted request re-enters it at the end at the step of its
+  promotion (key 2 a_i for an arrival, 2 t + 1 for a promotion at step t, so promotions follow the
+  arrivals of the same step; simultaneous promotions in index order).  The length estimate starts
+  at l_i.  At the start of a step, an active request that has generated its estimate of tokens
+  without finishing (it then has more than l_i tokens to go) is removed, its tokens discarded,
+  its estimate set to u_i, and it is appended to the queue, eligible in the same step.  The text
+  says "more than l tokens"; running a request past its estimate would use memory the feasibility
+  check did not reserve, so the removal happens as soon as the estimate is used up ("as soon as
+  the currently served request generates l tokens", Section 5).  Promotions count as evictions.
+  The paper states A_ell for the two-point family o in {l, u}; with per-request intervals it uses
+  each request's own l_i and u_i.  Like A_max it needs s_i + u_i <= M.
 * Arrivals (an extension: the paper has all a_i = 0).  Request i is eligible from step a_i on;
   when nothing is active or eligible, time jumps to the next arrival.  Makespan = max C_i.
 * Step cap.  A run that has processed ``step_cap`` batches without finishing stops with status
@@ -50,8 +66,8 @@ from __future__ import annotations
 
 from typing import Sequence
 
-AMAX, AMIN, HSF = 0, 1, 2
-POLICY_NAMES = {AMAX: "A_max", AMIN: "A_min", HSF: "H-SF"}
+AMAX, AMIN, HSF, AR, AELL = 0, 1, 2, 3, 4
+POLICY_NAMES = {AMAX: "A_max", AMIN: "A_min", HSF: "H-SF", AR: "A_r", AELL: "A_ell"}
 
 OK, E_INVAL, E_INFEASIBLE, E_STEPCAP = 0, -1, -2, -3
 
@@ -62,15 +78,20 @@ def default_step_cap(o: Sequence[int]) -> int:
     return 64 * (len(o) + sum(int(x) for x in o))
 
 
-def validate(policy: int, M: int, a, s, l, u, o) -> int:
-    """Per-instance input check: 1 <= l <= o <= u, s >= 1, a >= 0, s + o <= M (s + u <= M for A_max)."""
+def validate(policy: int, M: int, a, s, l, u, o, rank=None) -> int:
+    """Per-instance input check: 1 <= l <= o <= u, s >= 1, a >= 0, rank >= 0 (A_r), s + o <= M
+    (s + u <= M for A_max and A_ell)."""
+    if policy not in POLICY_NAMES or (policy == AR and rank is None):
+        return E_INVAL
     for i in range(len(o)):
         if s[i] < 1 or a[i] < 0 or l[i] < 1 or l[i] > o[i] or o[i] > u[i]:
+            return E_INVAL
+        if policy == AR and rank[i] < 0:
             return E_INVAL
     for i in range(len(o)):
         if s[i] + o[i] > M:
             return E_INFEASIBLE
-        if policy == AMAX and s[i] + u[i] > M:
+        if policy in (AMAX, AELL) and s[i] + u[i] > M:
             return E_INFEASIBLE
     return OK
 
@@ -81,11 +102,13 @@ def _empty_result(status: int, n: int) -> dict:
 
 
 def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
-             refine: str = "max", same_step: bool = True, trace: list | None = None) -> dict:
+             refine: str = "max", same_step: bool = True, trace: list | None = None,
+             rank: Sequence[int] | None = None) -> dict:
     """Run one instance; return the result record plus per-request completion steps.
 
     ``trace`` (optional list) receives one dict per processed step: t, the batch, the admitted
-    and the evicted request indices, and the step's memory.
+    and the evicted (A_min) or promoted (A_ell) request indices, and the step's memory.
+    ``rank`` is A_r's permutation (rank[i] = position of request i), required for A_r only.
     """
     n = len(o)
     a = [int(x) for x in a]
@@ -93,7 +116,8 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
     l = [int(x) for x in l]
     u = [int(x) for x in u]
     o = [int(x) for x in o]
-    st = validate(policy, M, a, s, l, u, o)
+    rank = None if rank is None else [int(x) for x in rank]
+    st = validate(policy, M, a, s, l, u, o, rank)
     if st != OK:
         return _empty_result(st, n)
     if n == 0:
@@ -103,7 +127,8 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
     state = [_WAITING] * n
     start = [None] * n  # last start p_i
     gen = [0] * n  # tokens generated since the last start, g_i
-    otil = list(l)  # õ_i, the running lower bound (A_min)
+    otil = list(l)  # õ_i: the running lower bound (A_min), the current estimate l_i or u_i (A_ell)
+    qkey = [2 * x for x in a]  # A_ell queue position: 2 a_i on arrival, 2 t + 1 after a promotion
     completion = [0] * n
 
     tel = makespan = peak = evictions = steps = request_steps = 0
@@ -112,14 +137,18 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
     n_done = 0
 
     def est_len(i: int) -> int:
-        if policy == HSF:
+        if policy in (HSF, AR):
             return o[i]
         if policy == AMAX:
             return u[i]
         return otil[i]
 
     def key(i: int) -> int:
-        return est_len(i)  # the sort key is the length estimate for all three policies
+        if policy == AR:
+            return rank[i]
+        if policy == AELL:
+            return qkey[i]
+        return est_len(i)  # A_max, A_min, H-SF: the sort key is the length estimate
 
     def feasible(active: list, new: list) -> bool:
         """eq. Constraint at every step t' from t to the last projected step (literal)."""
@@ -175,6 +204,22 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
                     waiting = waiting + evicted
                     waiting = [i for i in range(n) if i in set(waiting)]
 
+        if policy == AELL:
+            # promote-l: a request that has used up its estimate without finishing leaves the
+            # batch, loses its tokens, takes u_i as its estimate and goes to the end of the queue
+            for i in active:
+                if gen[i] == otil[i]:
+                    otil[i] = u[i]
+                    gen[i] = 0
+                    start[i] = None
+                    state[i] = _WAITING
+                    qkey[i] = 2 * t + 1
+                    evictions += 1
+                    evicted.append(i)
+            if evicted:
+                active = [i for i in active if state[i] == _ACTIVE]
+                waiting = waiting + evicted
+
         waiting.sort(key=lambda i: (key(i), i))
         admitted = []
         for i in waiting:
@@ -208,6 +253,9 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
         if policy == AMIN:
             for i in batch:
                 assert otil[i] <= o[i]
+        if policy == AELL:
+            for i in batch:
+                assert gen[i] <= otil[i]
         if trace is not None:
             trace.append(dict(t=t, batch=sorted(batch), admitted=list(admitted),
                               evicted=list(evicted), finished=sorted(finished), mem=mem))

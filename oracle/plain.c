@@ -1,5 +1,6 @@
 /*
- * Plain CPU oracle of the batched schedulers A_max, A_min and H-SF (endpoint evaluation).
+ * Plain CPU oracle of the batched schedulers A_max, A_min, H-SF, A_r and A_ell (endpoint
+ * evaluation).
  *
  * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the CPU-baseline leg of
  * bench.py may load this library.  It shares no code, header, table or helper with the CUDA path.
@@ -10,7 +11,10 @@
  * Algorithm malb; the running lower bound for A_min, Algorithms milb / milbrevise), admission of
  * the largest feasible prefix of the waiting set sorted by (key, index), and A_min's
  * overflow eviction in ascending (lower bound, index) order with the refinement
- * lower_bound <- max(lower_bound, tokens generated).
+ * lower_bound <- max(lower_bound, tokens generated).  A_r (Algorithm random): true lengths and a
+ * given permutation rank as the queue key.  A_ell (Algorithm promote_l): FIFO queue (key 2 a_i on
+ * arrival, 2 t + 1 on re-entry at step t), estimate l_i, and at the start of a step a request that
+ * has used up its estimate unfinished is removed, takes u_i and re-enters at the end.
  *
  * The only difference from the literal oracle is how the constraint is checked: instead of
  * every future step t', it is checked at the projected last steps ("endpoints") of the jobs.
@@ -26,7 +30,7 @@
 #include <stdlib.h>
 #include <string.h>
 
-enum { O_AMAX = 0, O_AMIN = 1, O_HSF = 2 };
+enum { O_AMAX = 0, O_AMIN = 1, O_HSF = 2, O_AR = 3, O_AELL = 4 };
 enum { O_OK = 0, O_E_INVAL = -1, O_E_INFEASIBLE = -2, O_E_STEPCAP = -3, O_E_NOMEM = -6 };
 
 typedef struct {
@@ -97,12 +101,15 @@ static int endpoints_fit(ep_t *buf, int32_t m, int64_t M) {
 
 /* ---- per-instance validation (Section 2 model; interface requirements) ------------------------ */
 static int validate(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
-                    const int32_t *l, const int32_t *u, const int32_t *o) {
-    for (int32_t i = 0; i < n; i++)
+                    const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank) {
+    if (policy == O_AR && !rank) return O_E_INVAL;
+    for (int32_t i = 0; i < n; i++) {
         if (s[i] < 1 || a[i] < 0 || l[i] < 1 || l[i] > o[i] || o[i] > u[i]) return O_E_INVAL;
+        if (policy == O_AR && rank[i] < 0) return O_E_INVAL;
+    }
     for (int32_t i = 0; i < n; i++) {
         if ((int64_t)s[i] + o[i] > M) return O_E_INFEASIBLE;
-        if (policy == O_AMAX && (int64_t)s[i] + u[i] > M) return O_E_INFEASIBLE;
+        if ((policy == O_AMAX || policy == O_AELL) && (int64_t)s[i] + u[i] > M) return O_E_INFEASIBLE;
     }
     return O_OK;
 }
@@ -137,18 +144,19 @@ int64_t oracle_default_step_cap(int32_t n, const int32_t *o) {
 /*
  * Simulate one instance.  step_cap <= 0 selects the default cap 64 * (n + sum o).
  * completion (optional, n entries) receives each request's completion step C_i.
+ * rank (A_r only; may be NULL otherwise) is the permutation position of each request.
  */
-int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
-               const int32_t *l, const int32_t *u, const int32_t *o, int64_t step_cap,
-               oracle_result *res, int64_t *completion) {
+int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+                  const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                  int64_t step_cap, oracle_result *res, int64_t *completion) {
     memset(res, 0, sizeof(*res));
     if (completion)
         for (int32_t i = 0; i < n; i++) completion[i] = 0;
-    if (policy < 0 || policy > 2 || n < 0) {
+    if (policy < 0 || policy > 4 || n < 0) {
         res->status = O_E_INVAL;
         return O_E_INVAL;
     }
-    int st = validate(policy, M, n, a, s, l, u, o);
+    int st = validate(policy, M, n, a, s, l, u, o, rank);
     if (st != O_OK || n == 0) {
         res->status = st;
         return st;
@@ -158,6 +166,7 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
     /* per-request state */
     int64_t *start = (int64_t *)malloc(sizeof(int64_t) * n);
     int32_t *otil = (int32_t *)malloc(sizeof(int32_t) * n);
+    int64_t *qkey = (int64_t *)malloc(sizeof(int64_t) * n);
     int32_t *act = (int32_t *)malloc(sizeof(int32_t) * n);
     int32_t *nxt = (int32_t *)malloc(sizeof(int32_t) * n);
     arr_t *arr = (arr_t *)malloc(sizeof(arr_t) * n);
@@ -167,14 +176,15 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
     heap_t q;
     q.v = (uint64_t *)malloc(sizeof(uint64_t) * n);
     q.n = 0;
-    if (!start || !otil || !act || !nxt || !arr || !ep || !tmp || !ev || !q.v) {
-        free(start); free(otil); free(act); free(nxt); free(arr); free(ep); free(tmp); free(ev);
-        free(q.v);
+    if (!start || !otil || !qkey || !act || !nxt || !arr || !ep || !tmp || !ev || !q.v) {
+        free(start); free(otil); free(qkey); free(act); free(nxt); free(arr); free(ep); free(tmp);
+        free(ev); free(q.v);
         res->status = O_E_NOMEM;
         return O_E_NOMEM;
     }
     for (int32_t i = 0; i < n; i++) {
         otil[i] = l[i];
+        qkey[i] = 2 * (int64_t)a[i];
         arr[i].a = a[i];
         arr[i].i = i;
     }
@@ -185,7 +195,8 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
     int64_t t = arr[0].a;
     int status = O_OK;
 
-#define EST(i) (policy == O_HSF ? o[i] : policy == O_AMAX ? u[i] : otil[i])
+#define EST(i) (policy == O_HSF || policy == O_AR ? o[i] : policy == O_AMAX ? u[i] : otil[i])
+#define QKEY(i) (policy == O_AR ? (uint32_t)rank[i] : policy == O_AELL ? (uint32_t)qkey[i] : (uint32_t)EST(i))
 
     while (n_done < n) {
         if (steps >= cap) {
@@ -195,7 +206,7 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
         /* arrivals: requests with a_i <= t join the waiting set */
         while (ap < n && arr[ap].a <= t) {
             int32_t i = (int32_t)arr[ap].i;
-            heap_push(&q, ((uint64_t)(uint32_t)EST(i) << 32) | (uint32_t)i);
+            heap_push(&q, ((uint64_t)QKEY(i) << 32) | (uint32_t)i);
             ap++;
         }
         if (an == 0 && q.n == 0) { /* idle: jump to the next arrival */
@@ -229,6 +240,24 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
                     if (start[act[k]] >= 0) act[m++] = act[k];
                 an = m;
             }
+        }
+
+        /* A_ell: a request that used up its estimate unfinished goes to the end of the queue */
+        if (policy == O_AELL) {
+            int32_t m = 0;
+            for (int32_t k = 0; k < an; k++) {
+                int32_t i = act[k];
+                if (t - start[i] == otil[i]) {
+                    otil[i] = u[i];
+                    start[i] = -1;
+                    qkey[i] = 2 * t + 1;
+                    evictions++;
+                    heap_push(&q, ((uint64_t)QKEY(i) << 32) | (uint32_t)i);
+                } else {
+                    act[m++] = i;
+                }
+            }
+            an = m;
         }
 
         /* admission: largest feasible prefix of the waiting set in (key, index) order */
@@ -282,6 +311,7 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
         steps++;
         t++;
     }
+#undef QKEY
 #undef EST
 
     res->total_latency = tel;
@@ -291,9 +321,15 @@ int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t
     res->steps = steps;
     res->request_steps = rsteps;
     res->status = status;
-    free(start); free(otil); free(act); free(nxt); free(arr); free(ep); free(tmp); free(ev);
-    free(q.v);
+    free(start); free(otil); free(qkey); free(act); free(nxt); free(arr); free(ep); free(tmp);
+    free(ev); free(q.v);
     return status;
+}
+
+int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+               const int32_t *l, const int32_t *u, const int32_t *o, int64_t step_cap,
+               oracle_result *res, int64_t *completion) {
+    return oracle_run_ex(policy, M, n, a, s, l, u, o, NULL, step_cap, res, completion);
 }
 
 /* ---- many instances (CSR), spread over threads ------------------------------------------------ */
@@ -302,7 +338,7 @@ typedef struct {
     int64_t M;
     int32_t n_inst;
     const int64_t *off;
-    const int32_t *a, *s, *l, *u, *o;
+    const int32_t *a, *s, *l, *u, *o, *rank;
     int64_t step_cap;
     oracle_result *res;
     int64_t *completion;
@@ -318,23 +354,23 @@ static void *batch_worker(void *arg) {
         pthread_mutex_unlock(&b->mu);
         if (i >= b->n_inst) break;
         int64_t lo = b->off[i], hi = b->off[i + 1];
-        oracle_run(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
-                   b->u + lo, b->o + lo, b->step_cap, &b->res[i],
-                   b->completion ? b->completion + lo : NULL);
+        oracle_run_ex(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
+                      b->u + lo, b->o + lo, b->rank ? b->rank + lo : NULL, b->step_cap, &b->res[i],
+                      b->completion ? b->completion + lo : NULL);
     }
     return NULL;
 }
 
-int oracle_run_batch(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
-                     const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
-                     const int32_t *o, int64_t step_cap, oracle_result *res, int64_t *completion,
-                     int32_t n_threads) {
+int oracle_run_batch_ex(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                        const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                        const int32_t *o, const int32_t *rank, int64_t step_cap, oracle_result *res,
+                        int64_t *completion, int32_t n_threads) {
     batch_t b;
     b.policy = policy;
     b.M = M;
     b.n_inst = n_inst;
     b.off = offsets;
-    b.a = a; b.s = s; b.l = l; b.u = u; b.o = o;
+    b.a = a; b.s = s; b.l = l; b.u = u; b.o = o; b.rank = rank;
     b.step_cap = step_cap;
     b.res = res;
     b.completion = completion;
@@ -353,4 +389,12 @@ int oracle_run_batch(int policy, int64_t M, int32_t n_inst, const int64_t *offse
     for (int32_t i = 0; i < n_inst; i++)
         if (res[i].status < worst) worst = res[i].status;
     return worst;
+}
+
+int oracle_run_batch(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                     const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                     const int32_t *o, int64_t step_cap, oracle_result *res, int64_t *completion,
+                     int32_t n_threads) {
+    return oracle_run_batch_ex(policy, M, n_inst, offsets, a, s, l, u, o, NULL, step_cap, res,
+                               completion, n_threads);
 }

@@ -51,6 +51,13 @@ def lib():
                                        i32p, i32p, i32p, ctypes.c_int64, ctypes.c_void_p, i64p,
                                        ctypes.c_int32]
         L.oracle_run_batch.restype = ctypes.c_int
+        L.oracle_run_ex.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i32p, i32p, i32p, i32p,
+                                    i32p, i32p, ctypes.c_int64, ctypes.c_void_p, i64p]
+        L.oracle_run_ex.restype = ctypes.c_int
+        L.oracle_run_batch_ex.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i64p, i32p, i32p,
+                                          i32p, i32p, i32p, i32p, ctypes.c_int64, ctypes.c_void_p, i64p,
+                                          ctypes.c_int32]
+        L.oracle_run_batch_ex.restype = ctypes.c_int
         L.oracle_default_step_cap.argtypes = [ctypes.c_int32, i32p]
         L.oracle_default_step_cap.restype = ctypes.c_int64
         _lib = L
@@ -61,7 +68,9 @@ def _i32(x) -> np.ndarray:
     return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
 
 
-def _p32(x: np.ndarray):
+def _p32(x: np.ndarray | None):
+    if x is None:
+        return ctypes.POINTER(ctypes.c_int32)()
     return x.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
 
 
@@ -71,14 +80,17 @@ def _p64(x: np.ndarray | None):
     return x.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
 
 
-def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool = False) -> dict:
-    """One instance.  Returns the result fields (and 'completion' if asked)."""
+def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool = False,
+        rank=None) -> dict:
+    """One instance.  Returns the result fields (and 'completion' if asked).  ``rank`` is A_r's
+    permutation (rank[i] = position of request i)."""
     a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
+    rank = None if rank is None else _i32(rank)
     n = int(o.shape[0])
     res = np.zeros(1, dtype=RESULT_DTYPE)
     comp = np.zeros(max(n, 1), dtype=np.int64) if completions else None
-    lib().oracle_run(int(policy), int(M), n, _p32(a), _p32(s), _p32(l), _p32(u), _p32(o),
-                     int(step_cap), res.ctypes.data, _p64(comp))
+    lib().oracle_run_ex(int(policy), int(M), n, _p32(a), _p32(s), _p32(l), _p32(u), _p32(o), _p32(rank),
+                        int(step_cap), res.ctypes.data, _p64(comp))
     out = {k: int(res[0][k]) for k in FIELDS}
     if completions:
         out["completion"] = comp[:n].tolist()
@@ -86,17 +98,18 @@ def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool
 
 
 def run_batch(policy: int, M: int, offsets, a, s, l, u, o, step_cap: int = 0, n_threads: int = 1,
-              completions: bool = False):
+              completions: bool = False, rank=None):
     """Many instances in CSR layout.  Returns a structured array (RESULT_DTYPE) and optionally the
     per-request completion steps."""
     offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
     a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
+    rank = None if rank is None else _i32(rank)
     n_inst = int(offsets.shape[0] - 1)
     res = np.zeros(n_inst, dtype=RESULT_DTYPE)
     comp = np.zeros(max(int(offsets[-1]), 1), dtype=np.int64) if completions else None
-    lib().oracle_run_batch(int(policy), int(M), n_inst, _p64(offsets), _p32(a), _p32(s), _p32(l),
-                           _p32(u), _p32(o), int(step_cap), res.ctypes.data, _p64(comp),
-                           int(n_threads))
+    lib().oracle_run_batch_ex(int(policy), int(M), n_inst, _p64(offsets), _p32(a), _p32(s), _p32(l),
+                              _p32(u), _p32(o), _p32(rank), int(step_cap), res.ctypes.data, _p64(comp),
+                              int(n_threads))
     if completions:
         return res, comp[: int(offsets[-1])]
     return res
@@ -105,7 +118,8 @@ def run_batch(policy: int, M: int, offsets, a, s, l, u, o, step_cap: int = 0, n_
 def run_workload(policy: int, w, step_cap: int = 0, n_threads: int = 1, completions: bool = False):
     """Convenience: run a ``Workload`` (from the seeded generator) through the C oracle."""
     return run_batch(policy, w.M, w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o,
-                     step_cap=step_cap, n_threads=n_threads, completions=completions)
+                     step_cap=step_cap, n_threads=n_threads, completions=completions,
+                     rank=w.ranks() if policy == 3 else None)
 
 
 def default_step_cap(o) -> int:

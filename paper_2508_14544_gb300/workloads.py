@@ -17,6 +17,10 @@ exactly (no float rounding).
 
 Per-instance seeding: instance i of a workload draws from ``numpy.random.default_rng(seed0 + i)``
 in the fixed order s, o, l, arrivals, so any subset of instances is reproducible on its own.
+
+The auxiliary policy A_r (Algorithm random) also needs a uniformly random permutation of each
+instance's requests; ``Workload.ranks()`` draws it from a separate stream,
+``numpy.random.default_rng([seed0 + i, 1])``, and returns rank[j] = position of request j.
 """
 from __future__ import annotations
 
@@ -51,6 +55,8 @@ class Workload:
     true_o: np.ndarray  # int32 [n_total]  o_i
     alpha: list = field(default_factory=list)  # per-instance Fraction
     instance_ids: np.ndarray | None = None  # global instance id of each row
+    seed0: int | None = None  # seed base of the named workload (for ranks())
+    _ranks: np.ndarray | None = None
 
     @property
     def n_instances(self) -> int:
@@ -71,6 +77,23 @@ class Workload:
             o=self.true_o[lo:hi],
         )
 
+    def ranks(self) -> np.ndarray:
+        """A_r's random permutation of every instance, as int32 ranks in CSR layout: rank[j] is the
+        position of request j in its instance's permutation.  Drawn per instance from
+        default_rng([seed0 + id, 1]) (instance id = global id when known, else the row)."""
+        if self._ranks is None:
+            out = np.zeros(self.n_total, dtype=np.int32)
+            base = 0 if self.seed0 is None else self.seed0
+            for r in range(self.n_instances):
+                lo, hi = int(self.offsets[r]), int(self.offsets[r + 1])
+                iid = r if self.instance_ids is None else int(self.instance_ids[r])
+                perm = np.random.default_rng([base + iid, 1]).permutation(hi - lo)
+                rk = np.empty(hi - lo, dtype=np.int32)
+                rk[perm] = np.arange(hi - lo, dtype=np.int32)
+                out[lo:hi] = rk
+            self._ranks = out
+        return self._ranks
+
     def uniform_n(self) -> int | None:
         d = np.diff(self.offsets)
         return int(d[0]) if d.size and np.all(d == d[0]) else None
@@ -78,7 +101,9 @@ class Workload:
     def subset(self, rows: Sequence[int]) -> "Workload":
         parts = [self.instance(int(i)) for i in rows]
         ids = None if self.instance_ids is None else self.instance_ids[np.asarray(rows, dtype=np.int64)]
-        return concat_instances(self.name, self.M, parts, [self.alpha[int(i)] for i in rows], ids)
+        w = concat_instances(self.name, self.M, parts, [self.alpha[int(i)] for i in rows], ids)
+        w.seed0 = self.seed0
+        return w
 
 
 def interval_for(o: np.ndarray, alpha: Fraction, rng: np.random.Generator) -> tuple[np.ndarray, np.ndarray]:
@@ -233,4 +258,6 @@ def make_workload(name: str, instances: Sequence[int] | range | None = None) -> 
     ids = range(spec.n_instances) if instances is None else instances
     ids = np.asarray(list(ids), dtype=np.int64)
     parts = [make_instance(name, int(i)) for i in ids]
-    return concat_instances(name, spec.M, parts, [p["alpha"] for p in parts], ids)
+    w = concat_instances(name, spec.M, parts, [p["alpha"] for p in parts], ids)
+    w.seed0 = spec.seed0
+    return w

@@ -1,7 +1,8 @@
 """Checks of an oracle implementation against values the paper and the mathematics fix.
 
-``check_all(sim)`` runs every pin against ``sim(policy, M, a, s, l, u, o) -> dict`` (a dict with
-the result fields and 'completion') and returns the list of failures.  The pin tests call it on
+``check_all(sim)`` runs every pin against ``sim(policy, M, a, s, l, u, o, rank=None) -> dict`` (a
+dict with the result fields and 'completion'; ``rank`` is A_r's permutation) and returns the list of
+failures.  The pin tests call it on
 both oracles; the mutation tests call it on deliberately broken copies of the literal oracle and
 expect failures.
 """
@@ -11,8 +12,8 @@ import json
 from pathlib import Path
 
 GOLDEN = Path(__file__).resolve().parent / "golden"
-AMAX, AMIN, HSF = 0, 1, 2
-POL = {"AMAX": AMAX, "AMIN": AMIN, "HSF": HSF}
+AMAX, AMIN, HSF, AR, AELL = 0, 1, 2, 3, 4
+POL = {"AMAX": AMAX, "AMIN": AMIN, "HSF": HSF, "AR": AR, "AELL": AELL}
 FIELDS = ("total_latency", "makespan", "peak_memory", "evictions", "steps", "request_steps")
 
 
@@ -57,6 +58,44 @@ def amax_wave_cases():
     return out
 
 
+def aell_wave_cases():
+    """A_ell on the two-point family (Algorithm promote_l): n = k*W requests with equal s, each of
+    length l or u (estimate l first), M = k(s+l) and M - k_u(s+u) <= s with k_u = floor(M/(s+u)).
+    First pass: FIFO waves of k, wave w runs steps w*l .. (w+1)*l - 1 and fills M exactly at its
+    last step, so nothing else starts meanwhile; its short requests complete at (w+1)*l, its long
+    ones have used up l unfinished and are promoted at step (w+1)*l behind all first-pass
+    requests.  Second pass, from W*l: the N_u long requests (estimate u = o) in promotion order,
+    waves of k_u lasting u steps (the slack below s+1 again lets nothing start inside a wave).
+    TEL = sum_short (w+1)*l + sum over long waves j of |wave_j| * (W*l + (j+1)*u); evictions =
+    N_u; request steps = n*l + N_u*u; steps = makespan = W*l + ceil(N_u/k_u)*u; peak = M."""
+    out = []
+    for (k, W, s, l, u, pattern) in [(4, 2, 1, 2, 5, "SLLSSLSL"), (2, 3, 3, 3, 9, "LSSLLS"),
+                                     (3, 3, 2, 4, 7, "SSLLSLSLL"), (4, 3, 1, 2, 5, "LLLLSSSSLSLS"),
+                                     (2, 2, 1, 3, 3, "SSSS")]:
+        n = k * W
+        assert len(pattern) == n
+        M = k * (s + l)
+        ku = M // (s + u)
+        assert ku >= 1 and M - ku * (s + u) <= s
+        o = [l if c == "S" else u for c in pattern]
+        tel, longs = 0, []
+        for w in range(W):
+            for i in range(w * k, (w + 1) * k):
+                if o[i] == l:
+                    tel += (w + 1) * l
+                else:
+                    longs.append(i)
+        nu = len(longs)
+        nw = -(-nu // ku)
+        for j in range(nw):
+            tel += min(ku, nu - j * ku) * (W * l + (j + 1) * u)
+        span = W * l + nw * u
+        exp = dict(total_latency=tel, makespan=span, peak_memory=M, evictions=nu, steps=span,
+                   request_steps=n * l + nu * u)
+        out.append(((k, W, s, l, u, pattern), M, [0] * n, [s] * n, [l] * n, [u] * n, o, exp))
+    return out
+
+
 def check_all(sim) -> list:
     fails = []
 
@@ -70,9 +109,9 @@ def check_all(sim) -> list:
             elif got.get(key) != val:
                 fails.append((tag, key, got.get(key), val))
 
-    def run(tag, *args):
+    def run(tag, *args, rank=None):
         try:
-            return sim(*args)
+            return sim(*args, rank=rank) if rank is not None else sim(*args)
         except AssertionError as e:  # an internal invariant tripped
             fails.append((tag, "assertion", str(e), None))
             return None
@@ -92,7 +131,8 @@ def check_all(sim) -> list:
     for name, case in ht.items():
         if name.startswith("_"):
             continue
-        r = run(name, POL[case["policy"]], case["M"], case["a"], case["s"], case["l"], case["u"], case["o"])
+        r = run(name, POL[case["policy"]], case["M"], case["a"], case["s"], case["l"], case["u"], case["o"],
+                rank=case.get("rank"))
         if r is not None:
             chk(name, r, case["expect"])
 
@@ -105,4 +145,16 @@ def check_all(sim) -> list:
         r = run(f"amaxwaves{tag}", AMAX, M, a, s, l, u, o)
         if r is not None:
             chk(f"amaxwaves{tag}", r, exp)
+    for tag, M, a, s, l, u, o, exp in aell_wave_cases():
+        r = run(f"aellwaves{tag}", AELL, M, a, s, l, u, o)
+        if r is not None:
+            chk(f"aellwaves{tag}", r, exp)
+    # exact waves with l = u = o: A_r in index order and A_ell (no long request) are plain FIFO
+    for tag, M, a, s, l, u, o, exp in wave_cases():
+        r = run(f"waves{tag}/AR", AR, M, a, s, l, u, o, rank=list(range(len(o))))
+        if r is not None:
+            chk(f"waves{tag}/AR", r, exp)
+        r = run(f"waves{tag}/AELL", AELL, M, a, s, l, u, o)
+        if r is not None:
+            chk(f"waves{tag}/AELL", r, exp)
     return fails

@@ -31,13 +31,18 @@ LIT_MUTATIONS = {
                          "new_bound = gen[i]"),
     "admit_longest_first": ("waiting.sort(key=lambda i: (key(i), i))", "waiting.sort(key=lambda i: (-key(i), i))"),
     "amax_uses_lower": ("        if policy == AMAX:\n            return u[i]", "        if policy == AMAX:\n            return l[i]"),
-    "hsf_uses_upper": ("        if policy == HSF:\n            return o[i]", "        if policy == HSF:\n            return u[i]"),
+    "hsf_uses_upper": ("        if policy in (HSF, AR):\n            return o[i]", "        if policy == AR:\n            return o[i]\n        if policy == HSF:\n            return u[i]"),
     "evict_trigger_without_plus_one": ("need = sum(s[i] + gen[i] + 1 for i in active)",
                                        "need = sum(s[i] + gen[i] for i in active)"),
     "completion_one_early": ("completion[i] = t + 1\n", "completion[i] = t\n"),
     "latency_from_start_zero": ("tel += t + 1 - a[i]", "tel += t - a[i]"),
     "evictee_waits": ("same_step: bool = True", "same_step: bool = False"),
     "peak_before_step": ("        mem = sum(s[i] + gen[i] for i in batch)", "        mem = sum(s[i] + gen[i] - 1 for i in batch)"),
+    "aell_promotion_ahead_of_arrivals": ("qkey[i] = 2 * t + 1", "qkey[i] = 2 * t - 1"),
+    "aell_keeps_lower_estimate": ("                    otil[i] = u[i]\n", "                    otil[i] = o[i] + 1\n"),
+    "aell_promotes_one_step_late": ("                if gen[i] == otil[i]:", "                if gen[i] == otil[i] + 1:"),
+    "ar_projects_upper": ("        if policy in (HSF, AR):\n            return o[i]", "        if policy == HSF:\n            return o[i]\n        if policy == AR:\n            return u[i]"),
+    "ar_ignores_rank": ("        if policy == AR:\n            return rank[i]", "        if policy == AR:\n            return o[i]"),
 }
 
 
@@ -52,13 +57,13 @@ def test_literal_mutation_is_caught(name):
     old, new = LIT_MUTATIONS[name]
     assert LIT.count(old) == 1, f"mutation anchor not found once: {name}"
     mod = _load_literal(LIT.replace(old, new))
-    fails = pins.check_all(lambda p, M, a, s, l, u, o: mod.simulate(p, M, a, s, l, u, o))
+    fails = pins.check_all(lambda p, M, a, s, l, u, o, rank=None: mod.simulate(p, M, a, s, l, u, o, rank=rank))
     assert fails, f"mutation {name} passed every pin"
 
 
 def test_unmutated_literal_passes():
     mod = _load_literal(LIT)
-    assert pins.check_all(lambda p, M, a, s, l, u, o: mod.simulate(p, M, a, s, l, u, o)) == []
+    assert pins.check_all(lambda p, M, a, s, l, u, o, rank=None: mod.simulate(p, M, a, s, l, u, o, rank=rank)) == []
 
 
 PLAIN_MUTATIONS = {
@@ -67,6 +72,9 @@ PLAIN_MUTATIONS = {
     "evict_need_no_plus_one": ("need += s[act[k]] + (t - start[act[k]]) + 1;", "need += s[act[k]] + (t - start[act[k]]);"),
     "no_clamp_for_amin": ("if (policy == O_AMIN && e < t) e = t;", "(void)0;"),
     "refine_to_tokens": ("if (g > otil[i]) otil[i] = (int32_t)g;", "otil[i] = (int32_t)g;"),
+    "aell_promotion_key_even": ("qkey[i] = 2 * t + 1;", "qkey[i] = 2 * t;"),
+    "aell_estimate_not_raised": ("                    otil[i] = u[i];\n", "                    otil[i] = o[i] + 1;\n"),
+    "ar_key_is_length": ("#define QKEY(i) (policy == O_AR ? (uint32_t)rank[i]", "#define QKEY(i) (policy == O_AR ? (uint32_t)o[i]"),
 }
 
 
@@ -79,17 +87,19 @@ def _build_plain(src: str, tmp_path: Path):
     L = ctypes.CDLL(str(so))
     i32p = ctypes.POINTER(ctypes.c_int32)
     i64p = ctypes.POINTER(ctypes.c_int64)
-    L.oracle_run.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i32p, i32p, i32p, i32p, i32p,
-                             ctypes.c_int64, ctypes.c_void_p, i64p]
+    L.oracle_run_ex.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i32p, i32p, i32p, i32p, i32p,
+                                i32p, ctypes.c_int64, ctypes.c_void_p, i64p]
     from oracle.plain import RESULT_DTYPE, FIELDS
 
-    def sim(p, M, a, s, l, u, o):
+    def sim(p, M, a, s, l, u, o, rank=None):
         arrs = [np.ascontiguousarray(np.asarray(v, np.int32)) for v in (a, s, l, u, o)]
+        rk = None if rank is None else np.ascontiguousarray(np.asarray(rank, np.int32))
         n = len(o)
         res = np.zeros(1, RESULT_DTYPE)
         comp = np.zeros(max(n, 1), np.int64)
-        L.oracle_run(p, M, n, *[x.ctypes.data_as(i32p) for x in arrs], 0, res.ctypes.data,
-                     comp.ctypes.data_as(i64p))
+        L.oracle_run_ex(p, M, n, *[x.ctypes.data_as(i32p) for x in arrs],
+                        rk.ctypes.data_as(i32p) if rk is not None else i32p(), 0, res.ctypes.data,
+                        comp.ctypes.data_as(i64p))
         out = {k: int(res[0][k]) for k in FIELDS}
         out["completion"] = comp[:n].tolist()
         return out

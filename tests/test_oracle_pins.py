@@ -6,8 +6,8 @@ from oracle import literal, plain
 from tests import pins
 
 SIMS = {
-    "literal": lambda p, M, a, s, l, u, o: literal.simulate(p, M, a, s, l, u, o),
-    "plain": lambda p, M, a, s, l, u, o: plain.run(p, M, a, s, l, u, o, completions=True),
+    "literal": lambda p, M, a, s, l, u, o, rank=None: literal.simulate(p, M, a, s, l, u, o, rank=rank),
+    "plain": lambda p, M, a, s, l, u, o, rank=None: plain.run(p, M, a, s, l, u, o, completions=True, rank=rank),
 }
 
 
