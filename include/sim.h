@@ -3,7 +3,7 @@
  *
  * The library simulates many independent instances of the single-worker LLM-inference
  * scheduling problem of arXiv 2508.14544 ("Adaptively Robust LLM Inference Optimization under
- * Prediction Uncertainty") on one GPU, under one of three policies:
+ * Prediction Uncertainty") on one GPU, under one of five policies:
  *
  *   SIM_AMAX - A_max, Algorithm malb (Section 3.2): every output length is taken to be its
  *              predicted upper bound u_i; each step admits the largest prefix of the waiting set,
@@ -16,6 +16,15 @@
  *              then admitted as for A_max, using the estimates.
  *   SIM_HSF  - the hindsight shortest-first benchmark H-SF, Algorithm off (Section 3.1, Appendix
  *              B): like A_max with the true output lengths.
+ *   SIM_AR   - the auxiliary policy A_r, Algorithm random (Appendix B): a fixed random permutation
+ *              of the requests (given by the caller as ranks, see sim_load_ranked_csr) and the true
+ *              output lengths; each step admits the largest feasible prefix in permutation order.
+ *   SIM_AELL - the promote-l policy A_ell, Algorithm promote_l (Section 5, two-point output
+ *              distributions; here with each request's own l_i and u_i): a FIFO waiting queue,
+ *              length estimate l_i; at the start of a step a job that has generated l_i tokens
+ *              without finishing is cancelled, takes u_i as its estimate and joins the end of the
+ *              queue (after the requests that arrived in that step; several in index order).
+ *              Each such promotion counts as a cancellation.  Steps must stay below 2^30.
  *
  * Model (Section 2): a worker with a KV cache of M tokens runs one batch per unit of time; every
  * member generates one token; a job's memory is its prompt size s_i plus the tokens generated so
@@ -39,12 +48,12 @@
 extern "C" {
 #endif
 
-typedef enum { SIM_AMAX = 0, SIM_AMIN = 1, SIM_HSF = 2 } sim_policy;
+typedef enum { SIM_AMAX = 0, SIM_AMIN = 1, SIM_HSF = 2, SIM_AR = 3, SIM_AELL = 4 } sim_policy;
 
 typedef enum {
     SIM_OK = 0,
     SIM_E_INVAL = -1,      /* bad argument, or an instance with l > o, o > u, l < 1, s < 1, a < 0 */
-    SIM_E_INFEASIBLE = -2, /* an instance has a request with s + o > M (or s + u > M under A_max) */
+    SIM_E_INFEASIBLE = -2, /* an instance has a request with s + o > M (or s + u > M under A_max, A_ell) */
     SIM_E_STEPCAP = -3,    /* an instance processed step_cap batches without finishing */
     SIM_E_CUDA = -4,       /* a CUDA runtime call failed; see sim_last_error */
     SIM_E_STATE = -5,      /* call out of order (e.g. sim_run before sim_load), or an internal check failed */
@@ -84,7 +93,7 @@ enum {
 /*
  * sim_create: set up a context for `n_instances` independent instances simulated under `policy`
  * with KV-cache limit M tokens (Section 2).
- *   policy      SIM_AMAX, SIM_AMIN or SIM_HSF.
+ *   policy      SIM_AMAX, SIM_AMIN, SIM_HSF, SIM_AR or SIM_AELL.
  *   M           1 <= M <= 2^26.
  *   n_instances >= 1.
  *   out         receives the new context (owned by the caller; free with sim_destroy).
@@ -108,7 +117,8 @@ int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out);
  * does not wait for other work on the device); the caller may free or reuse its arrays as soon as
  * the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
  * the call: they are reported in that instance's sim_result.status by sim_run.
- * Returns SIM_OK, SIM_E_INVAL (n_per_instance < 0, null pointer), SIM_E_NOMEM or SIM_E_CUDA.
+ * Returns SIM_OK, SIM_E_INVAL (n_per_instance < 0, null pointer; under SIM_AR, which needs
+ * sim_load_ranked_csr), SIM_E_NOMEM or SIM_E_CUDA.
  */
 int sim_load(sim_ctx *ctx, int32_t n_per_instance, const int32_t *arrival_t, const int32_t *prompt_s,
              const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o, int device_ptrs);
@@ -121,6 +131,19 @@ int sim_load(sim_ctx *ctx, int32_t n_per_instance, const int32_t *arrival_t, con
  */
 int sim_load_csr(sim_ctx *ctx, const int64_t *offsets, const int32_t *arrival_t, const int32_t *prompt_s,
                  const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o, int device_ptrs);
+
+/*
+ * sim_load_ranked_csr: sim_load_csr plus the random permutation that Algorithm random (A_r,
+ * Appendix B) draws before it starts; the draw is the caller's, so runs are reproducible.
+ *   rank   int32 per request, same layout and memory kind as the other arrays: rank_i >= 0 is the
+ *          position of request i in its instance's permutation (a permutation of 0..n-1 is the
+ *          intended use; equal ranks are ordered by request index).  Required (non-NULL) under
+ *          SIM_AR; ignored under the other policies.
+ * A negative rank makes that instance SIM_E_INVAL.  Returns as sim_load_csr.
+ */
+int sim_load_ranked_csr(sim_ctx *ctx, const int64_t *offsets, const int32_t *arrival_t, const int32_t *prompt_s,
+                        const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o,
+                        const int32_t *rank, int device_ptrs);
 
 /*
  * sim_run: simulate every loaded instance and write n_instances results to `out` (HOST memory).
@@ -158,7 +181,8 @@ int64_t sim_kernel_launches(const sim_ctx *ctx);
  * would fail or fragment that reservation), or a latency-sensitive loop that must avoid the
  * implicitly synchronising allocation calls (cudaFree waits for the whole device).
  * Semantics and results are those of sim_load_csr + sim_run with default options.
- *   policy, M, n_instances  as for sim_create (1 <= n_instances <= 16384).
+ *   policy, M, n_instances  as for sim_create, policy SIM_AMAX, SIM_AMIN or SIM_HSF
+ *               (1 <= n_instances <= 16384).
  *   offsets     HOST, n_instances + 1 int64, as for sim_load_csr.
  *   arrival_t .. true_o     DEVICE int32 arrays (current device), layout as for sim_load_csr.
  *   results     DEVICE, n_instances sim_result, written by the kernels.

@@ -13,7 +13,7 @@ import numpy as np
 
 from .build import LIB
 
-SIM_AMAX, SIM_AMIN, SIM_HSF = 0, 1, 2
+SIM_AMAX, SIM_AMIN, SIM_HSF, SIM_AR, SIM_AELL = 0, 1, 2, 3, 4
 SIM_OK, SIM_E_INVAL, SIM_E_INFEASIBLE, SIM_E_STEPCAP, SIM_E_CUDA, SIM_E_STATE, SIM_E_NOMEM = 0, -1, -2, -3, -4, -5, -6
 SIM_OPT_STEP_CAP, SIM_OPT_RECORD_COMPLETIONS, SIM_OPT_WARPS_PER_BLOCK, SIM_OPT_SMEM_ACTIVE_CAP = 1, 2, 3, 4
 SIM_OPT_WARPS_PER_SM = 5
@@ -34,7 +34,7 @@ RESULT_DTYPE = np.dtype([
 ])
 assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
 
-EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
+EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_load_ranked_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
            "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc")
 
 _lib = None
@@ -67,6 +67,8 @@ def lib() -> ctypes.CDLL:
     L.sim_load.restype = ctypes.c_int
     L.sim_load_csr.argtypes = [vp, vp, vp, vp, vp, vp, vp, ctypes.c_int]
     L.sim_load_csr.restype = ctypes.c_int
+    L.sim_load_ranked_csr.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, ctypes.c_int]
+    L.sim_load_ranked_csr.restype = ctypes.c_int
     L.sim_run.argtypes = [vp, vp, vp]
     L.sim_run.restype = ctypes.c_int
     L.sim_get_completions.argtypes = [vp, vp]
@@ -123,6 +125,12 @@ def sim_load_csr(ctx, offsets: np.ndarray, a, s, l, u, o, device_ptrs: int) -> i
     assert offsets.dtype == np.int64 and offsets.flags.c_contiguous
     return lib().sim_load_csr(ctx, offsets.ctypes.data, _ptr(a), _ptr(s), _ptr(l), _ptr(u), _ptr(o),
                               int(device_ptrs))
+
+
+def sim_load_ranked_csr(ctx, offsets: np.ndarray, a, s, l, u, o, rank, device_ptrs: int) -> int:
+    assert offsets.dtype == np.int64 and offsets.flags.c_contiguous
+    return lib().sim_load_ranked_csr(ctx, offsets.ctypes.data, _ptr(a), _ptr(s), _ptr(l), _ptr(u), _ptr(o),
+                                     _ptr(rank) if rank is not None else None, int(device_ptrs))
 
 
 def sim_run(ctx, out: np.ndarray, stream: int = 0) -> int:

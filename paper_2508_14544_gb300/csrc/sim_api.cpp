@@ -40,7 +40,8 @@ struct sim_ctx {
     int32_t n_max = 0;
     // device buffers
     int64_t *d_off = nullptr;
-    int32_t *d_raw = nullptr;  // 5 * cap_total
+    int32_t *d_raw = nullptr;  // 6 * cap_total: a, s, l, u, o, rank
+    int2 *d_lu = nullptr;      // A_ell: (l, u) per request, cap_total
     int64_t cap_total = 0;
     QEnt *d_rec = nullptr;
     int32_t *d_rec_a = nullptr;
@@ -120,7 +121,7 @@ extern "C" {
 int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out) {
     if (!out) return fail(nullptr, SIM_E_INVAL, "sim_create: out is NULL");
     *out = nullptr;
-    if (policy < SIM_AMAX || policy > SIM_HSF) return fail(nullptr, SIM_E_INVAL, "sim_create: bad policy %d", policy);
+    if (policy < SIM_AMAX || policy > SIM_AELL) return fail(nullptr, SIM_E_INVAL, "sim_create: bad policy %d", policy);
     if (M < 1 || M > simgb::kMaxM)
         return fail(nullptr, SIM_E_INVAL, "sim_create: M=%lld outside [1, 2^26]", (long long)M);
     if (n_instances < 1) return fail(nullptr, SIM_E_INVAL, "sim_create: n_instances=%d < 1", n_instances);
@@ -164,8 +165,8 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
     }
 }
 
-int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int32_t *s, const int32_t *l,
-                 const int32_t *u, const int32_t *o, int device_ptrs) {
+static int load_impl(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int32_t *s, const int32_t *l,
+                     const int32_t *u, const int32_t *o, const int32_t *rank, int device_ptrs) {
     if (!c) return SIM_E_INVAL;
     c->err.clear();
     c->loaded = false;
@@ -182,14 +183,17 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
     }
     const int64_t nt = offsets[c->n_inst];
     if (nt > 0 && (!a || !s || !l || !u || !o)) return fail(c, SIM_E_INVAL, "sim_load: NULL input array");
+    if (c->policy == SIM_AR && nt > 0 && !rank)
+        return fail(c, SIM_E_INVAL, "sim_load: A_r needs the permutation ranks (sim_load_ranked_csr)");
     int rc = check_device(c);
     if (rc) return rc;
     cudaError_t e;
     if (nt > c->cap_total || !c->d_raw) {
         const int64_t cap = std::max<int64_t>(nt, 1);
-        if ((e = dalloc(c->d_raw, size_t(5) * cap * sizeof(int32_t))) != cudaSuccess ||
+        if ((e = dalloc(c->d_raw, size_t(6) * cap * sizeof(int32_t))) != cudaSuccess ||
             (e = dalloc(c->d_rec, size_t(cap) * sizeof(QEnt))) != cudaSuccess ||
-            (e = dalloc(c->d_rec_a, size_t(cap) * sizeof(int32_t))) != cudaSuccess) {
+            (e = dalloc(c->d_rec_a, size_t(cap) * sizeof(int32_t))) != cudaSuccess ||
+            (c->policy == SIM_AELL && (e = dalloc(c->d_lu, size_t(cap) * sizeof(int2))) != cudaSuccess)) {
             c->cap_total = 0;
             return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_load: device allocation failed")
                                                   : cuda_fail(c, e, "cudaMalloc");
@@ -210,8 +214,9 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
         return cuda_fail(c, e, "sim_load: stream creation");
     const cudaStream_t ls = c->load_stream;
     const cudaMemcpyKind kind = device_ptrs ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
-    const int32_t *src[5] = {a, s, l, u, o};
-    for (int k = 0; k < 5; ++k) {
+    const int32_t *src[6] = {a, s, l, u, o, rank};
+    const int nsrc = (c->policy == SIM_AR) ? 6 : 5;
+    for (int k = 0; k < nsrc; ++k) {
         if (nt == 0) break;
         e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t), kind, ls);
         if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the input arrays");
@@ -229,6 +234,8 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
     sp.l = c->d_raw + 2 * c->cap_total;
     sp.u = c->d_raw + 3 * c->cap_total;
     sp.o = c->d_raw + 4 * c->cap_total;
+    sp.rank = c->d_raw + 5 * c->cap_total;
+    sp.lu = c->d_lu;
     sp.rec = c->d_rec;
     sp.rec_a = c->d_rec_a;
     sp.info = c->d_info;
@@ -241,6 +248,17 @@ int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int
     c->n_max = int32_t(n_max);
     c->loaded = true;
     return SIM_OK;
+}
+
+int sim_load_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int32_t *s, const int32_t *l,
+                 const int32_t *u, const int32_t *o, int device_ptrs) {
+    return load_impl(c, offsets, a, s, l, u, o, nullptr, device_ptrs);
+}
+
+int sim_load_ranked_csr(sim_ctx *c, const int64_t *offsets, const int32_t *a, const int32_t *s,
+                        const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                        int device_ptrs) {
+    return load_impl(c, offsets, a, s, l, u, o, rank, device_ptrs);
 }
 
 int sim_load(sim_ctx *c, int32_t n, const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
@@ -313,6 +331,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.info = c->d_info;
     p.res = c->d_res;
     p.completion = c->record_completions ? c->d_comp : nullptr;
+    p.lu = c->d_lu;
     p.ca = ca;
     p.dcap = dcap;
     p.use_smem = smem ? 1 : 0;
@@ -433,6 +452,7 @@ void sim_destroy(sim_ctx *c) {
     if (!c) return;
     dfree(c->d_off);
     dfree(c->d_raw);
+    dfree(c->d_lu);
     dfree(c->d_rec);
     dfree(c->d_rec_a);
     dfree(c->d_info);

@@ -10,10 +10,13 @@ namespace simgb {
 // the host re-runs such instances with a larger, global-memory workspace.
 constexpr int32_t kStatusCapacity = -100;
 constexpr int64_t kMaxM = int64_t(1) << 26;
+// A_ell queue keys are 2 a (arrival) and 2 t + 1 (promotion at step t): steps stay below 2^30.
+constexpr int32_t kAellMaxStep = (int32_t(1) << 30) - 1;
 
 // One waiting request as the queue stores it; queues are ordered by (key, idx).
 struct QEnt {
-    int32_t key;  // length estimate used as the sort key: u (A_max), o (H-SF), current lower bound (A_min)
+    int32_t key;  // sort key: u (A_max), o (H-SF), current lower bound (A_min), permutation rank
+                  // (A_r), queue position 2 a / 2 t + 1 (A_ell)
     int32_t idx;  // request index within its instance
     int32_t s;    // prompt size
     int32_t o;    // true output length
@@ -41,7 +44,9 @@ struct StageParams {
     int64_t step_cap;          // 0: default 64 * (n + sum o)
     const int64_t *off;        // n_inst + 1
     const int32_t *a, *s, *l, *u, *o;  // raw copies, n_total each
+    const int32_t *rank;       // A_r: permutation rank per request (n_total), else unused
     QEnt *rec;                 // out: per instance, sorted by (a, key, idx)
+    int2 *lu;                  // out (A_ell only, else null): (l, u) of request idx at base + idx
     int32_t *rec_a;            // out: arrival step of rec[i]
     InstInfo *info;            // out: n_inst
 };
@@ -56,6 +61,7 @@ struct RunParams {
     const InstInfo *info;
     DevResult *res;
     int64_t *completion;       // optional, n_total
+    const int2 *lu;            // A_ell: (l, u) per request (staged), else null
     // workspace
     int32_t ca;                // active-set capacity per instance (multiple of 32)
     int32_t dcap;              // delta-queue capacity per instance (multiple of 32)

@@ -10,6 +10,10 @@
 //       every future step (Algorithms malb / milb / off);
 //   S6  process the batch: one token per member, the step's memory sum(s + tokens) (eq.
 //       constraintM), completions, TEL (eq. latency).
+// Two more policies share the loop: A_r (Algorithm random: the queue key is a given permutation
+// rank, the projected length the true o) and A_ell (Algorithm promote_l: FIFO queue, estimate l;
+// at the start of a step a job that used up its estimate unfinished is removed, takes u and
+// re-enters the queue at its end; the queue key is 2 a on arrival and 2 t + 1 on re-entry).
 //
 // Active set (per warp, shared memory; a global-memory workspace of the same layout serves
 // instances that outgrow it), structure of arrays sorted by the projected last step E:
@@ -45,7 +49,7 @@ namespace simgb {
 namespace {
 
 constexpr unsigned FULL = 0xffffffffu;
-enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
+enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2, P_AR = 3, P_AELL = 4 };
 enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
 constexpr int kChunk = 128;  // active-set entries per warp pass (4 per lane)
 constexpr int kWin = 32;     // admission window (one candidate per lane)
@@ -56,6 +60,19 @@ __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 
 __device__ __forceinline__ bool qless(const QEnt &a, const QEnt &b) {
     return a.key < b.key || (a.key == b.key && a.idx < b.idx);
+}
+
+// The admission code reads an entry's key as its projected length.  For A_max, A_min and H-SF the
+// sort key is that length; A_r projects the true length o and A_ell the current estimate (l before
+// a promotion, u after: promotions have odd keys).
+template <int POL>
+__device__ __forceinline__ QEnt proj(const RunParams &P, int64_t base, QEnt e) {
+    if (POL == P_AR) e.key = e.o;
+    if (POL == P_AELL) {
+        const int2 lu = P.lu[base + e.idx];
+        e.key = (e.key & 1) ? lu.y : lu.x;
+    }
+    return e;
 }
 
 __device__ __forceinline__ int sat32(int64_t v) {
@@ -716,6 +733,72 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     return W;
 }
 
+// Largest admissible prefix when the window is in queue order but not in length order (A_r: the
+// permutation, A_ell: the FIFO queue).  Candidate c reaches a point x iff its last step
+// t + L_c - 1 >= x, so every point keeps its own sum: the active endpoints' projected memory is kept
+// in the K array (these policies do not use it) and each window entry m accumulates, in a register,
+// the candidates so far whose length is >= L_m (itself included); entry m's point counts once m is
+// admitted.  Any active-set size.
+__device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int tb, int SB0, int64_t M, int t,
+                                                         int W, const QEnt &mine) {
+    const int lane = lane_id();
+    const int Mi = int(M);
+    for (int j = lane; j < A; j += 32) {
+        const int ej = w.E[j];
+        w.K[j] = (ej >= t) ? sat32(int64_t(w.SB[j]) + int64_t(A - j) * (int64_t(ej) - tb)) : INT_MIN;
+    }
+    const int Lm = mine.key, dm = Lm - 1;
+    int av = 0, acc = 0;
+    if (lane < W) {
+        const int64_t y = int64_t(t) + dm;
+        const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
+        av = sat32(int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb));
+    }
+    int64_t need = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
+    for (int k = 1; k <= W; ++k) {
+        const int c = k - 1;
+        const int sc = __shfl_sync(FULL, mine.s, c) + 1;
+        const int Lc = __shfl_sync(FULL, mine.key, c);
+        need += sc;
+        bool fail = false;
+        for (int j = lane; j < A; j += 32) {  // each lane updates only its own points
+            const int v = w.K[j];
+            const int dj = w.E[j] - t;
+            if (v != INT_MIN && Lc > dj) {
+                const int nv = v + sc + dj;
+                w.K[j] = nv;
+                fail = fail || nv > Mi;
+            }
+        }
+        if (lane < W && Lc >= Lm) acc += sc + dm;
+        if (lane <= c) fail = fail || int64_t(av) + acc > M;
+        if (__ballot_sync(FULL, fail) != 0 || need > M) return k - 1;
+    }
+    return W;
+}
+
+// Order the K admitted window entries by projected length (the active set is sorted by the last
+// step E = t + L - 1); equal lengths keep their queue order.
+__device__ __forceinline__ void sort_admitted(const Ws &w, int K, QEnt &mine) {
+    const int lane = lane_id();
+    int rk = 0;
+    for (int m = 0; m < K; ++m) {
+        const int Lo = __shfl_sync(FULL, mine.key, m);
+        rk += (Lo < mine.key || (Lo == mine.key && m < lane)) ? 1 : 0;
+    }
+    __syncwarp();
+    if (lane < K) w.cnt[rk] = lane;  // the merge histogram is free here
+    __syncwarp();
+    const int src = lane < K ? w.cnt[lane] : lane;
+    __syncwarp();
+    QEnt o;
+    o.key = __shfl_sync(FULL, mine.key, src);
+    o.idx = __shfl_sync(FULL, mine.idx, src);
+    o.s = __shfl_sync(FULL, mine.s, src);
+    o.o = __shfl_sync(FULL, mine.o, src);
+    if (lane < K) mine = o;
+}
+
 // First step tau in (t, tau_lim) at which the head candidate (prompt s, estimate L) fits, with the
 // active set unchanged; kBig if none.  In terms of y = tau + L - 1, the interval between active
 // endpoints (E[j-1], E[j]] has #{E < y} = j, and #{E <= y} = j below E[j] and the end of E[j]'s
@@ -891,11 +974,37 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 continue;
             }
         }
+        // ---- A_ell: jobs that used up their estimate unfinished (E < t; the set is sorted by E, so
+        // they lead it) leave the batch and re-enter the queue at its end with the estimate u
+        if (POL == P_AELL && A > 0 && w.E[0] < t) {
+            if (t > kAellMaxStep) {
+                status = ST_STEPCAP;
+                break;
+            }
+            const int c = warp_prefix_count(A, [&](int i) { return w.E[i] < t; });
+            for (int j = 0; j < c; ++j) {  // in position order; the delta orders equal keys by index
+                const int b = w.B[j], p = w.P[j], f = w.F[j], id = w.I[j];
+                QEnt e;
+                e.key = 2 * t + 1;
+                e.idx = id;
+                e.s = b + p - 1;
+                e.o = f - p + 1;
+                __syncwarp();
+                if (lane == 0) w.F[j] = -1;
+                __syncwarp();
+                delta_insert(w, q, e);
+            }
+            nev += c;
+            tb_next = t;
+            pend_compact = true;
+            hvalid = false;
+            continue;
+        }
         // ---- S4/S5: admit the largest feasible prefix of R_t
         for (;;) {
             if (!hvalid) {
                 if (queue_empty(q)) break;
-                h = queue_head(w, q);
+                h = proj<POL>(P, info.base, queue_head(w, q));
                 hvalid = true;
                 pdirty = true;
             }
@@ -926,7 +1035,12 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             mine.key = mine.idx = mine.s = mine.o = 0;
             int msrc = 0;
             const int W = build_window(w, q, mine, msrc);
-            const int Kadm = admissible_prefix(w, A, tb, SB0, M, t, W, mine);
+            if (POL == P_AR || POL == P_AELL) {
+                if (lane < W) mine = proj<POL>(P, info.base, mine);
+            }
+            const int Kadm = (POL == P_AR || POL == P_AELL)
+                                 ? admissible_prefix_general(w, A, tb, SB0, M, t, W, mine)
+                                 : admissible_prefix(w, A, tb, SB0, M, t, W, mine);
             if (Kadm <= 0) {
                 status = ST_STATE;  // the head test and the window disagree: internal error
                 break;
@@ -934,6 +1048,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             const int cm = __popc(__ballot_sync(FULL, lane < Kadm && msrc == 0));
             q.mh += cm;
             q.dn -= Kadm - cm;
+            // entries >= Kadm stay in their lanes, so the new head below is unaffected
+            if ((POL == P_AR || POL == P_AELL) && Kadm > 1) sort_admitted(w, Kadm, mine);
             if (!insert_window(w, A, Kadm, t, mine)) {
                 status = kStatusCapacity;
                 break;
@@ -986,6 +1102,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             int64_t tau = nextF;
             if (ap < n) tau = min(tau, int64_t(next_a));
             if (POL == P_AMIN && A > 0) tau = min(tau, int64_t(tb) + floor_div32(M - SB0, A) + 1);
+            if (POL == P_AELL && A > 0) tau = min(tau, int64_t(w.E[0]) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
             if (tau > int64_t(t) + 1 && hvalid && A > 0)
                 tau = min(tau, first_fit_step(w, A, tb, SB0, M, t, h.s, h.key, tau));
@@ -1046,8 +1163,11 @@ const void *run_fn(bool smem) {
 size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
-    const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true) : policy == P_AMIN ? run_fn<P_AMIN>(true)
-                                                                                : run_fn<P_HSF>(true);
+    const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true)
+                     : policy == P_AMIN ? run_fn<P_AMIN>(true)
+                     : policy == P_HSF  ? run_fn<P_HSF>(true)
+                     : policy == P_AR   ? run_fn<P_AR>(true)
+                                        : run_fn<P_AELL>(true);
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
 }
 
@@ -1064,9 +1184,17 @@ cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per
             if (sm) k_run<P_AMIN, true><<<grid, block, smem_bytes, st>>>(p);
             else k_run<P_AMIN, false><<<grid, block, smem_bytes, st>>>(p);
             break;
-        default:
+        case P_HSF:
             if (sm) k_run<P_HSF, true><<<grid, block, smem_bytes, st>>>(p);
             else k_run<P_HSF, false><<<grid, block, smem_bytes, st>>>(p);
+            break;
+        case P_AR:
+            if (sm) k_run<P_AR, true><<<grid, block, smem_bytes, st>>>(p);
+            else k_run<P_AR, false><<<grid, block, smem_bytes, st>>>(p);
+            break;
+        default:
+            if (sm) k_run<P_AELL, true><<<grid, block, smem_bytes, st>>>(p);
+            else k_run<P_AELL, false><<<grid, block, smem_bytes, st>>>(p);
             break;
     }
     return cudaGetLastError();

@@ -135,6 +135,8 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     sp.l = lower_l;
     sp.u = upper_u;
     sp.o = true_o;
+    sp.rank = nullptr;
+    sp.lu = nullptr;
     sp.rec = d_rec;
     sp.rec_a = d_rec_a;
     sp.info = d_info;
@@ -153,6 +155,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.info = d_info;
     p.res = reinterpret_cast<simgb::DevResult *>(results);
     p.completion = nullptr;
+    p.lu = nullptr;
     p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
     p.dcap = kNaDeltaCap;
     p.use_smem = 0;

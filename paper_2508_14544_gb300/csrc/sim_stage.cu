@@ -5,7 +5,9 @@
 //              constants the simulation needs (sum of arrivals for TEL, the step cap), and sort
 //              the requests by (arrival step, policy key, index) so that every arrival batch is
 //              already in the order of the waiting set R_t (key u for Algorithm malb, l for
-//              Algorithms milb / milbrevise, o for Algorithm off).
+//              Algorithms milb / milbrevise, o for Algorithm off, the given permutation rank for
+//              Algorithm random, and the FIFO position 2 a for Algorithm promote_l, which also
+//              gets its (l, u) table).
 //   k_ratio  - per instance TEL(pi) / TEL(H-SF) in IEEE double (Definition cr).
 #include <climits>
 #include <cstdint>
@@ -17,7 +19,7 @@ namespace simgb {
 namespace {
 
 constexpr unsigned FULL = 0xffffffffu;
-enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2 };
+enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2, P_AR = 3, P_AELL = 4 };
 enum { ST_OK = 0, ST_INVAL = -1, ST_INFEASIBLE = -2 };
 
 __device__ __forceinline__ bool stage_less(int aa, const QEnt &x, int ab, const QEnt &y) {
@@ -53,8 +55,20 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
         const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
         if (s < 1 || a < 0 || l < 1 || l > o || o > u) bad_inval = 1;
         if (int64_t(s) + o > S.M) bad_inf = 1;
-        if (S.policy == P_AMAX && int64_t(s) + u > S.M) bad_inf = 1;
-        const int key = (S.policy == P_AMAX) ? u : (S.policy == P_HSF ? o : l);
+        if ((S.policy == P_AMAX || S.policy == P_AELL) && int64_t(s) + u > S.M) bad_inf = 1;
+        int key;
+        switch (S.policy) {
+            case P_AMAX: key = u; break;
+            case P_HSF: key = o; break;
+            case P_AR: key = S.rank[g]; break;
+            case P_AELL: key = 2 * min(a, kAellMaxStep); break;
+            default: key = l; break;
+        }
+        if (S.policy == P_AR && key < 0) bad_inval = 1;
+        if (S.policy == P_AELL) {
+            if (a > kAellMaxStep) bad_inval = 1;
+            S.lu[g] = make_int2(l, u);  // indexed by request: j == idx below
+        }
         QEnt e;
         e.key = key;
         e.idx = j;

@@ -31,12 +31,13 @@ def main(argv=None) -> None:
     w = W.make_workload(args.workload, ids)
     import torch
     dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
+    rank = torch.from_numpy(w.ranks()).cuda() if POLICIES[args.policy] == 3 else None
     opts = {}
     if args.warps_per_block:
         opts["warps_per_block"] = args.warps_per_block
     with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
         for _ in range(args.repeat):
-            sim.load(w.offsets, *dev)
+            sim.load(w.offsets, *dev, rank=rank)
             torch.cuda.synchronize()
             t0 = time.perf_counter()
             res = sim.run()

@@ -35,19 +35,27 @@ class Simulator:
             raise L.SimError(rc, L.sim_last_error(self.ctx))
         return rc
 
-    def load(self, offsets, a, s, l, u, o) -> None:
+    def load(self, offsets, a, s, l, u, o, rank=None) -> None:
+        """Load requests (host numpy arrays or CUDA int32 tensors).  ``rank`` is A_r's permutation
+        (same layout and memory kind); when given, sim_load_ranked_csr is used."""
         offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
         dev = hasattr(a, "is_cuda") and a.is_cuda
+        src = (a, s, l, u, o) if rank is None else (a, s, l, u, o, rank)
         if dev:
-            arrs = [x.contiguous() for x in (a, s, l, u, o)]
+            arrs = [x.contiguous() for x in src]
             for x in arrs:
                 assert str(x.dtype) == "torch.int32"
         else:
-            arrs = [_i32_host(x) for x in (a, s, l, u, o)]
-        self._check(L.sim_load_csr(self.ctx, offsets, *arrs, 1 if dev else 0))
+            arrs = [_i32_host(x) for x in src]
+        if rank is None:
+            self._check(L.sim_load_csr(self.ctx, offsets, *arrs, 1 if dev else 0))
+        else:
+            self._check(L.sim_load_ranked_csr(self.ctx, offsets, *arrs, 1 if dev else 0))
 
     def load_workload(self, w) -> None:
-        self.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o)
+        """Load a seeded ``Workload``; under A_r its ranks() are the permutation."""
+        rank = w.ranks() if self.policy == L.SIM_AR else None
+        self.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o, rank=rank)
 
     def run(self, stream: int = 0) -> np.ndarray:
         out = np.zeros(self.n_instances, dtype=L.RESULT_DTYPE)

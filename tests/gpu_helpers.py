@@ -12,15 +12,21 @@ def n_threads() -> int:
     return max(1, min(32, os.cpu_count() or 1))
 
 
-def gpu_run(policy, w, device_load=True, completions=False, **opts):
+def gpu_run(policy, w, device_load=True, completions=False, rank=None, **opts):
+    """A_r (policy 3) takes ``rank`` or, if None, the workload's own ranks()."""
     import torch
 
     from paper_2508_14544_gb300 import Simulator
+    if policy == 3 and rank is None:
+        rank = w.ranks()
     with Simulator(policy, w.M, w.n_instances, record_completions=int(completions), **opts) as sim:
         if device_load:
             dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in
                    (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
-            sim.load(w.offsets, *dev)
+            rk = None if rank is None else torch.from_numpy(np.ascontiguousarray(np.asarray(rank, np.int32))).cuda()
+            sim.load(w.offsets, *dev, rank=rk)
+        elif rank is not None:
+            sim.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o, rank=np.asarray(rank, np.int32))
         else:
             sim.load_workload(w)
         res = sim.run()

@@ -7,7 +7,7 @@ from tests.gpu_helpers import FIELDS, assert_same, gpu_run, oracle_run
 
 pytestmark = pytest.mark.gpu
 
-POLS = (0, 1, 2)
+POLS = (0, 1, 2, 3, 4)  # A_max, A_min, H-SF, A_r, A_ell
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -19,17 +19,18 @@ def _cuda():
     g.build()
 
 
-def _gpu_sim(p, M, a, s, l, u, o):
+def _gpu_sim(p, M, a, s, l, u, o, rank=None):
     from paper_2508_14544_gb300 import workloads as W
     w = W.concat_instances("pin", M, [dict(a=a, s=s, l=l, u=u, o=o)])
-    res, comp = gpu_run(p, w, completions=True)
+    res, comp = gpu_run(p, w, completions=True, rank=rank)
     out = {k: int(res[0][k]) for k in FIELDS}
     out["completion"] = comp.tolist()
     return out
 
 
 def test_paper_pins_on_gpu():
-    """Example 1, the Definition-1 example, the hand traces and the wave closed forms."""
+    """Example 1, the Definition-1 example, the hand traces (A_min, A_ell, A_r) and the wave closed
+    forms (all policies, and A_ell's two-pass waves)."""
     fails = pins.check_all(_gpu_sim)
     assert not fails, fails
 
@@ -127,9 +128,15 @@ def test_c4_full_sampled(pol):
     assert np.all(got["status"] == 0)
     assert np.all(got["peak_memory"] <= w.M)
     so = np.add.reduceat(w.true_o.astype(np.int64), w.offsets[:-1])
-    if pol in (0, 2):
+    if pol in (0, 2, 3):
         assert np.all(got["evictions"] == 0)
         assert np.array_equal(got["request_steps"], so)
+    elif pol == 4:
+        # promote-l: every request with o > l is promoted exactly once, wasting l tokens
+        longer = w.true_o > w.lower
+        assert np.array_equal(got["evictions"], np.add.reduceat(longer.astype(np.int64), w.offsets[:-1]))
+        wasted = np.add.reduceat(np.where(longer, w.lower, 0).astype(np.int64), w.offsets[:-1])
+        assert np.array_equal(got["request_steps"], so + wasted)
     else:
         assert np.all(got["request_steps"] >= so)
 
