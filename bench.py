@@ -189,7 +189,7 @@ def run_ours(args) -> None:
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2508_14544_gb300 import SIM_AMAX, SIM_AMIN, SIM_HSF, Simulator
+    from paper_2508_14544_gb300 import SIM_AELL, SIM_AMAX, SIM_AMIN, SIM_AR, SIM_HSF, Simulator
 
     rank, world, local = dist_env()
     if world > 1:
@@ -275,6 +275,29 @@ def run_ours(args) -> None:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
     e2e_val = rs_per_step * e2e_steps * world / e2e_s
+
+    # the paper's two further policies on the same instances (outside the step): A_r (Algorithm
+    # random, permutation drawn by the workload generator) and A_ell (Algorithm promote_l);
+    # sim_run device time by CUDA events, median of 3 after a warm-up
+    further = {}
+    for name, pol in (("A_r", SIM_AR), ("A_ell", SIM_AELL)):
+        with Simulator(pol, w.M, w.n_instances) as sim:
+            rk = torch.from_numpy(w.ranks()).to(dev) if pol == SIM_AR else None
+            sim.load(w.offsets, *d_in, rank=rk)
+            r = sim.run(sh)
+            assert np.all(r["status"] == 0), (name, r["status"])
+            ms = []
+            for _ in range(3):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record(stream)
+                sim.run(sh)
+                e1.record(stream)
+                torch.cuda.synchronize()
+                ms.append(e0.elapsed_time(e1))
+        rsn = int(r["request_steps"].sum())
+        further[name] = {"sim_run_ms": round(statistics.median(ms), 3), "request_steps": rsn,
+                         "request_steps_per_s": rsn / (statistics.median(ms) / 1000.0)}
     h2d = 3 * 5 * w.n_total * 4
     d2h = 3 * w.n_instances * 56 + 2 * w.n_instances * 8
 
@@ -299,7 +322,8 @@ def run_ours(args) -> None:
                    "parallelism": f"instances sharded, {world} replica(s), no collective on the data path",
                    "l2": "256 MB buffer written between timed steps (inputs are 20 MB < L2)",
                    "request_steps_per_step": rs_per_step,
-                   "sim_run_ms": dict(zip(POLICY_NAMES, [round(x, 3) for x in per_pol_ms]))},
+                   "sim_run_ms": dict(zip(POLICY_NAMES, [round(x, 3) for x in per_pol_ms])),
+                   "further_policies_not_in_step": further},
         "roofline": {"bound": "alu", "kernel": f"k_run<{POLICY_NAMES[dom]}>",
                      "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12,
                      "unit": "Tops/s (int32)", "frac": achieved_ops / peak_ops,
