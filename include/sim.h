@@ -201,6 +201,36 @@ int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const int64_t *o
                     const int32_t *prompt_s, const int32_t *lower_l, const int32_t *upper_u, const int32_t *true_o,
                     sim_result *results, void *cuda_stream);
 
+/*
+ * sim_cr_amin_lemma: the large-M competitive ratio of A_min given by Lemma thm:Amin (Section 4.1)
+ * for a batch of output-length histograms, in IEEE double.  Every request has prompt size s and
+ * an output length in [l, u], u = l + len - 1; histogram h gives x_k, the fraction (or count) of
+ * requests of length k, at x[h * len + (k - l)].
+ *   CR = sum_k d(k) S1(k) (d(k) S2(k) + 2 G(k)) / sum_k k (s+k) x_k (x_k + 2 sum_{i>k} x_i),
+ *   d(l) = s + l, d(k) = 1 otherwise, S1(k) = sum_{i>=k} i x_i, S2(k) = sum_{i>=k} x_i / (s+i),
+ *   G(k) = sum_{i>k} (i-k) x_i / (s+i).
+ *   n_hist     >= 0 histograms; len >= 1; l >= 1; s >= 0.
+ *   x, cr_out  n_hist * len and n_hist doubles; HOST memory (device_ptrs = 0: the call copies,
+ *              computes and returns with the results in cr_out) or DEVICE memory of the current
+ *              device (device_ptrs = 1: the call only enqueues the kernel on cuda_stream).
+ * Entries must be >= 0 with a positive denominator (at least one x_k > 0); otherwise the ratio is
+ * not a number.  Returns SIM_OK, SIM_E_INVAL (message in sim_last_error(NULL)), SIM_E_NOMEM,
+ * SIM_E_CUDA.  No counterpart needs a context.
+ */
+int sim_cr_amin_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *cr_out,
+                      int device_ptrs, void *cuda_stream);
+
+/*
+ * sim_cr_amin_rho: for each u, the spectral radius of B_u^{-1} A_u (Corollary A/B, s = 0, l = 1:
+ * a_ij = min(i,j)^2/(ij) ((i+j)^2/2 - min(i,j)^2), b_ij = min(i,j)^2), the largest value of the
+ * Rayleigh quotient x'A_u x / x'B_u x and thus the bound on CR(A_min) of Section 4.1 (<= H_u).
+ *   u_values  HOST, n_u values in [1, 2^20];  rho_out  HOST, n_u doubles.
+ * Power iteration in double on the current device, synchronous; converges to the relative
+ * precision of double in well under 200 iterations (the second eigenvalue is below a third of the
+ * first for every u tried).  Returns SIM_OK, SIM_E_INVAL, SIM_E_NOMEM or SIM_E_CUDA.
+ */
+int sim_cr_amin_rho(int32_t n_u, const int32_t *u_values, double *rho_out);
+
 /* sim_set_option: set one of the SIM_OPT_* options.  Returns SIM_OK or SIM_E_INVAL. */
 int sim_set_option(sim_ctx *ctx, int key, int64_t value);
 

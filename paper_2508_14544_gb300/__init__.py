@@ -7,7 +7,7 @@ synthetic workload generator.
 """
 from ._lib import (SIM_AMAX, SIM_AMIN, SIM_HSF, SIM_AR, SIM_AELL, RESULT_DTYPE, SimError, lib, sim_create, sim_load,
                    sim_load_csr, sim_load_ranked_csr, sim_run, sim_get_completions, sim_competitive_ratio, sim_set_option, sim_last_error, sim_destroy,
-                   sim_kernel_launches)
+                   sim_kernel_launches, cr_amin_lemma, cr_amin_rho)
 from .sim import Simulator
 
 POLICIES = {"A_max": SIM_AMAX, "A_min": SIM_AMIN, "H-SF": SIM_HSF, "A_r": SIM_AR, "A_ell": SIM_AELL}

@@ -35,7 +35,8 @@ RESULT_DTYPE = np.dtype([
 assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
 
 EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_load_ranked_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
-           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc")
+           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc",
+           "sim_cr_amin_lemma", "sim_cr_amin_rho")
 
 _lib = None
 
@@ -85,6 +86,11 @@ def lib() -> ctypes.CDLL:
     L.sim_kernel_launches.restype = ctypes.c_int64
     L.sim_run_noalloc.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, vp, vp, vp, vp, vp, vp, vp, vp]
     L.sim_run_noalloc.restype = ctypes.c_int
+    L.sim_cr_amin_lemma.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_double, vp, vp,
+                                    ctypes.c_int, vp]
+    L.sim_cr_amin_lemma.restype = ctypes.c_int
+    L.sim_cr_amin_rho.argtypes = [ctypes.c_int32, vp, vp]
+    L.sim_cr_amin_rho.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -163,3 +169,35 @@ def sim_run_noalloc(policy: int, M: int, offsets: np.ndarray, a, s, l, u, o, res
 
 def sim_destroy(ctx) -> None:
     lib().sim_destroy(ctx)
+
+
+def cr_amin_lemma(x, l: int, s: float, stream: int = 0):
+    """Lemma thm:Amin for each row of ``x`` (host float64 array [n_hist, len] or a CUDA float64
+    tensor; a tensor gives a tensor, computed asynchronously on ``stream``)."""
+    if hasattr(x, "is_cuda") and x.is_cuda:
+        import torch
+        x = x.contiguous()
+        assert x.dtype == torch.float64 and x.dim() == 2
+        out = torch.empty(x.shape[0], dtype=torch.float64, device=x.device)
+        rc = lib().sim_cr_amin_lemma(int(x.shape[0]), int(x.shape[1]), int(l), float(s), x.data_ptr(),
+                                     out.data_ptr(), 1, ctypes.c_void_p(stream or None))
+    else:
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+        if x.ndim == 1:
+            x = x[None, :]
+        out = np.zeros(x.shape[0], dtype=np.float64)
+        rc = lib().sim_cr_amin_lemma(int(x.shape[0]), int(x.shape[1]), int(l), float(s), x.ctypes.data,
+                                     out.ctypes.data, 0, ctypes.c_void_p(stream or None))
+    if rc != SIM_OK:
+        raise SimError(rc, sim_last_error(None))
+    return out
+
+
+def cr_amin_rho(u_values) -> np.ndarray:
+    """Spectral radius of B_u^{-1} A_u for each u (Corollary A/B)."""
+    us = np.ascontiguousarray(np.asarray(u_values, dtype=np.int32).ravel())
+    out = np.zeros(us.shape[0], dtype=np.float64)
+    rc = lib().sim_cr_amin_rho(int(us.shape[0]), us.ctypes.data, out.ctypes.data)
+    if rc != SIM_OK:
+        raise SimError(rc, sim_last_error(None))
+    return out

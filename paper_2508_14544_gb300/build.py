@@ -13,7 +13,7 @@ CSRC = PKG / "csrc"
 INCLUDE = ROOT / "include"
 BUILD = PKG / "_build"
 LIB = BUILD / "libsim.so"
-SOURCES = ["sim_kernels.cu", "sim_stage.cu", "sim_api.cpp", "sim_noalloc.cu"]
+SOURCES = ["sim_kernels.cu", "sim_stage.cu", "sim_api.cpp", "sim_noalloc.cu", "sim_analytic.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -467,4 +467,78 @@ void sim_destroy(sim_ctx *c) {
     delete c;
 }
 
+/* ---- analytic competitive ratios (Lemma thm:Amin, Corollary A/B) --------------------------- */
+
+int sim_cr_amin_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *cr_out,
+                      int device_ptrs, void *cuda_stream) {
+    if (n_hist < 0 || len < 1 || l < 1 || !(s >= 0.0) || int64_t(l) + len - 1 > INT32_MAX)
+        return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_lemma: need n_hist >= 0, len >= 1, l >= 1, s >= 0");
+    if (n_hist == 0) return SIM_OK;
+    if (!x || !cr_out) return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_lemma: NULL x or cr_out");
+    cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+    cudaError_t e;
+    if (device_ptrs) {
+        e = simgb::launch_lemma(n_hist, len, l, s, x, cr_out, st);
+        if (e != cudaSuccess) return cuda_fail(nullptr, e, "sim_cr_amin_lemma: kernel launch");
+        return SIM_OK;
+    }
+    double *dx = nullptr, *dout = nullptr;
+    const size_t nx = size_t(n_hist) * size_t(len);
+    if ((e = cudaMalloc(&dx, nx * sizeof(double))) != cudaSuccess ||
+        (e = cudaMalloc(&dout, size_t(n_hist) * sizeof(double))) != cudaSuccess) {
+        cudaFree(dx);
+        return e == cudaErrorMemoryAllocation ? fail(nullptr, SIM_E_NOMEM, "sim_cr_amin_lemma: device allocation")
+                                              : cuda_fail(nullptr, e, "sim_cr_amin_lemma: cudaMalloc");
+    }
+    int rc = SIM_OK;
+    if ((e = cudaMemcpyAsync(dx, x, nx * sizeof(double), cudaMemcpyHostToDevice, st)) != cudaSuccess ||
+        (e = simgb::launch_lemma(n_hist, len, l, s, dx, dout, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(cr_out, dout, size_t(n_hist) * sizeof(double), cudaMemcpyDeviceToHost, st)) !=
+            cudaSuccess ||
+        (e = cudaStreamSynchronize(st)) != cudaSuccess)
+        rc = cuda_fail(nullptr, e, "sim_cr_amin_lemma");
+    cudaFree(dx);
+    cudaFree(dout);
+    return rc;
+}
+
+int sim_cr_amin_rho(int32_t n_u, const int32_t *u_values, double *rho_out) {
+    if (n_u < 0) return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_rho: n_u < 0");
+    if (n_u == 0) return SIM_OK;
+    if (!u_values || !rho_out) return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_rho: NULL argument");
+    int32_t umax = 0;
+    for (int32_t k = 0; k < n_u; ++k) {
+        if (u_values[k] < 1 || u_values[k] > (1 << 20))
+            return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_rho: u_values[%d]=%d outside [1, 2^20]", k, u_values[k]);
+        umax = std::max(umax, u_values[k]);
+    }
+    // batches of at most 256 MB of vectors (3 u doubles per value)
+    const int64_t stride = 3 * int64_t(umax);
+    const int64_t per_batch = std::max<int64_t>(1, (int64_t(256) << 20) / (stride * int64_t(sizeof(double))));
+    const int32_t nb = int32_t(std::min<int64_t>(per_batch, n_u));
+    double *scratch = nullptr, *dout = nullptr;
+    int32_t *dus = nullptr;
+    cudaError_t e;
+    if ((e = cudaMalloc(&scratch, size_t(nb) * size_t(stride) * sizeof(double))) != cudaSuccess ||
+        (e = cudaMalloc(&dout, size_t(nb) * sizeof(double))) != cudaSuccess ||
+        (e = cudaMalloc(&dus, size_t(nb) * sizeof(int32_t))) != cudaSuccess) {
+        cudaFree(scratch);
+        cudaFree(dout);
+        return e == cudaErrorMemoryAllocation ? fail(nullptr, SIM_E_NOMEM, "sim_cr_amin_rho: device allocation")
+                                              : cuda_fail(nullptr, e, "sim_cr_amin_rho: cudaMalloc");
+    }
+    int rc = SIM_OK;
+    for (int32_t b = 0; b < n_u && rc == SIM_OK; b += nb) {
+        const int32_t m = std::min(nb, n_u - b);
+        if ((e = cudaMemcpy(dus, u_values + b, size_t(m) * sizeof(int32_t), cudaMemcpyHostToDevice)) != cudaSuccess ||
+            (e = simgb::launch_rho(m, dus, dout, scratch, stride, 200, nullptr)) != cudaSuccess ||
+            (e = cudaMemcpy(rho_out + b, dout, size_t(m) * sizeof(double), cudaMemcpyDeviceToHost)) != cudaSuccess)
+            rc = cuda_fail(nullptr, e, "sim_cr_amin_rho");
+    }
+    cudaFree(scratch);
+    cudaFree(dout);
+    cudaFree(dus);
+    return rc;
+}
+
 }  // extern "C"

@@ -79,5 +79,9 @@ cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per
                        cudaStream_t st);
 cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
 cudaError_t set_run_smem_limit(int policy, size_t bytes);
+cudaError_t launch_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *out,
+                         cudaStream_t st);
+cudaError_t launch_rho(int32_t n_u, const int32_t *us, double *out, double *scratch, int64_t stride,
+                       int32_t max_iter, cudaStream_t st);
 
 }  // namespace simgb
