@@ -298,6 +298,26 @@ def run_ours(args) -> None:
         rsn = int(r["request_steps"].sum())
         further[name] = {"sim_run_ms": round(statistics.median(ms), 3), "request_steps": rsn,
                          "request_steps_per_s": rsn / (statistics.median(ms) / 1000.0)}
+
+    # the Lemma-thm:Amin evaluator on 2^20 histograms of 64 lengths (512 MB of doubles, read once):
+    # 20 FP64 flops per length (6 FMA + 8 other), so GB300's FP64 rate bounds it, not HBM
+    from paper_2508_14544_gb300 import cr_amin_lemma
+    hx = torch.rand((1 << 20, 64), dtype=torch.float64, device=dev)
+    for _ in range(3):
+        cr_amin_lemma(hx, 1, 0.0, stream=sh)
+    lm = []
+    for _ in range(5):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        cr_amin_lemma(hx, 1, 0.0, stream=sh)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        lm.append(e0.elapsed_time(e1))
+    lemma_bytes = hx.numel() * 8 + hx.shape[0] * 8
+    lemma_gbs = lemma_bytes / (statistics.median(lm) / 1000.0) / 1e9
+    lemma_tflops = 20.0 * hx.numel() / (statistics.median(lm) / 1000.0) / 1e12
+    del hx
     h2d = 3 * 5 * w.n_total * 4
     d2h = 3 * w.n_instances * 56 + 2 * w.n_instances * 8
 
@@ -323,7 +343,12 @@ def run_ours(args) -> None:
                    "l2": "256 MB buffer written between timed steps (inputs are 20 MB < L2)",
                    "request_steps_per_step": rs_per_step,
                    "sim_run_ms": dict(zip(POLICY_NAMES, [round(x, 3) for x in per_pol_ms])),
-                   "further_policies_not_in_step": further},
+                   "further_policies_not_in_step": further,
+                   "lemma_evaluator": {"histograms": 1 << 20, "lengths": 64, "ms": round(statistics.median(lm), 4),
+                                       "GB_per_s": round(lemma_gbs, 1),
+                                       "frac_of_measured_hbm": round(lemma_gbs / float(_peaks().get("hbm_gbs", 6800.0)), 3),
+                                       "fp64_tflops": round(lemma_tflops, 3),
+                                       "frac_of_nominal_fp64_1.25": round(lemma_tflops / 1.25, 3)}},
         "roofline": {"bound": "alu", "kernel": f"k_run<{POLICY_NAMES[dom]}>",
                      "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12,
                      "unit": "Tops/s (int32)", "frac": achieved_ops / peak_ops,

@@ -209,7 +209,7 @@ int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const int64_t *o
  *   CR = sum_k d(k) S1(k) (d(k) S2(k) + 2 G(k)) / sum_k k (s+k) x_k (x_k + 2 sum_{i>k} x_i),
  *   d(l) = s + l, d(k) = 1 otherwise, S1(k) = sum_{i>=k} i x_i, S2(k) = sum_{i>=k} x_i / (s+i),
  *   G(k) = sum_{i>k} (i-k) x_i / (s+i).
- *   n_hist     >= 0 histograms; len >= 1; l >= 1; s >= 0.
+ *   n_hist     >= 0 histograms; 1 <= len <= 8192; l >= 1; s >= 0.
  *   x, cr_out  n_hist * len and n_hist doubles; HOST memory (device_ptrs = 0: the call copies,
  *              computes and returns with the results in cr_out) or DEVICE memory of the current
  *              device (device_ptrs = 1: the call only enqueues the kernel on cuda_stream).

@@ -1,9 +1,10 @@
 // Analytic competitive-ratio evaluators of A_min (double precision, sm_103a).
 //
-//   k_lemma   - Lemma thm:Amin for a batch of length histograms: one warp per histogram walks it
-//               from the longest length down, keeping the suffix sums the lemma needs as warp
-//               scans (sum i x_i, sum x_i/(s+i), sum i x_i/(s+i), sum x_i over i >= k), so each
-//               histogram is read once: O(u) work, HBM-bound for large batches.
+//   k_lemma   - Lemma thm:Amin for a batch of length histograms: one thread per histogram walks it
+//               from the longest length down with the four running sums the lemma needs
+//               (sum i x_i, sum x_i/(s+i), sum i x_i/(s+i), sum x_i over i >= k), about ten FP64
+//               operations per length, with 1/(s+k) and k(s+k) from a shared-memory table.  The
+//               histogram is read once; GB300's FP64 rate, not HBM, bounds the kernel.
 //   k_rho     - spectral radius of B_u^{-1} A_u (Corollary A/B; s = 0, l = 1), the bound on the
 //               Rayleigh quotient of Section 4.1, by power iteration.  A_u v is O(u) from prefix
 //               and suffix sums (for j <= i, a_ij = ij/2 + j^2 - j^3/(2i); symmetric), B_u^{-1} is
@@ -28,17 +29,6 @@ __device__ __forceinline__ double warp_sum(double v) {
     return v;
 }
 
-// Inclusive suffix sum over lanes (lane i gets sum of lanes >= i).
-__device__ __forceinline__ double suffix_incl(double v) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-        const double y = __shfl_down_sync(FULL, v, d);
-        if (lane + d < 32) v += y;
-    }
-    return v;
-}
-
 // Inclusive prefix sum over lanes.
 __device__ __forceinline__ double prefix_incl(double v) {
     const int lane = threadIdx.x & 31;
@@ -50,49 +40,39 @@ __device__ __forceinline__ double prefix_incl(double v) {
     return v;
 }
 
-__global__ void k_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *__restrict__ x,
-                        double *__restrict__ out) {
-    const int lane = threadIdx.x & 31;
-    const int64_t warp = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = (int64_t(gridDim.x) * blockDim.x) >> 5;
-    for (int64_t h = warp; h < n_hist; h += nwarps) {
-        const double *xh = x + h * int64_t(len);
-        // carries: sums over lengths beyond the current chunk
-        double c_ix = 0.0, c_fr = 0.0, c_ifr = 0.0, c_x = 0.0;
-        double num = 0.0, den = 0.0;
-        const int nchunk = (len + 31) >> 5;
-        for (int c = nchunk - 1; c >= 0; --c) {
-            const int j = c * 32 + lane;  // index into the histogram, length k = l + j
-            const double k = double(l + j);
-            const double xk = (j < len) ? xh[j] : 0.0;
-            const double fr = xk / (s + k);
-            const double S1 = suffix_incl(k * xk) + c_ix;        // sum_{i>=k} i x_i
-            const double S2 = suffix_incl(fr) + c_fr;            // sum_{i>=k} x_i/(s+i)
-            const double T = suffix_incl(k * fr) + c_ifr;        // sum_{i>=k} i x_i/(s+i)
-            const double X = suffix_incl(xk) + c_x;              // sum_{i>=k} x_i
-            // values at k + 1 (from the next lane; the last lane takes the carry).  Every lane
-            // executes the shuffles; only the selection depends on the lane.
-            const double S2d = __shfl_down_sync(FULL, S2, 1);
-            const double Td = __shfl_down_sync(FULL, T, 1);
-            const double Xd = __shfl_down_sync(FULL, X, 1);
-            const double S2n = (lane == 31) ? c_fr : S2d;
-            const double Tn = (lane == 31) ? c_ifr : Td;
-            const double Xn = (lane == 31) ? c_x : Xd;
-            if (j < len) {
-                const double delta = (j == 0) ? (s + double(l)) : 1.0;
-                const double gap = Tn - k * S2n;                 // sum_{i>k} (i-k) x_i/(s+i)
-                num += delta * S1 * (delta * S2 + 2.0 * gap);
-                den += k * (s + k) * xk * (xk + 2.0 * Xn);
-            }
-            c_ix = __shfl_sync(FULL, S1, 0);
-            c_fr = __shfl_sync(FULL, S2, 0);
-            c_ifr = __shfl_sync(FULL, T, 0);
-            c_x = __shfl_sync(FULL, X, 0);
-        }
-        num = warp_sum(num);
-        den = warp_sum(den);
-        if (lane == 0) out[h] = num / den;
+__global__ void __launch_bounds__(256) k_lemma(int32_t n_hist, int32_t len, int32_t l, double s,
+                                                const double *__restrict__ x, double *__restrict__ out) {
+    // per-length constants shared by every histogram: 1/(s+k) and k(s+k)
+    extern __shared__ double tab[];
+    double *rinv = tab, *ck = tab + len;
+    for (int j = threadIdx.x; j < len; j += blockDim.x) {
+        const double k = double(l + j);
+        rinv[j] = 1.0 / (s + k);
+        ck[j] = k * (s + k);
     }
+    __syncthreads();
+    const int64_t h = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (h >= n_hist) return;
+    const double *xh = x + h * int64_t(len);
+    // running sums over lengths > k (before the update) and >= k (after it)
+    double S1 = 0.0, S2 = 0.0, T = 0.0, X = 0.0;
+    double num = 0.0, den = 0.0;
+    for (int j = len - 1; j >= 0; --j) {
+        const double k = double(l + j);
+        const double xk = __ldg(xh + j);
+        // values over i > k
+        const double gap = fma(-k, S2, T);      // sum_{i>k} (i-k) x_i/(s+i)
+        const double twoXn = 2.0 * X;           // 2 sum_{i>k} x_i
+        const double fr = xk * rinv[j];
+        S1 = fma(k, xk, S1);                    // sum_{i>=k} i x_i
+        S2 += fr;                               // sum_{i>=k} x_i/(s+i)
+        T = fma(k, fr, T);                      // sum_{i>=k} i x_i/(s+i)
+        X += xk;
+        const double delta = (j == 0) ? (s + double(l)) : 1.0;
+        num = fma(delta * S1, fma(2.0, gap, delta * S2), num);
+        den = fma(ck[j] * xk, xk + twoXn, den);
+    }
+    out[h] = num / den;
 }
 
 // (A v)_i and (B v)_i for i = 1..u from prefix/suffix sums; v, av, bv in global scratch.
@@ -195,12 +175,12 @@ __global__ void k_rho(int32_t n_u, const int32_t *__restrict__ us, double *__res
 cudaError_t launch_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *out,
                          cudaStream_t st) {
     if (n_hist <= 0) return cudaSuccess;
-    int dev = 0, n_sm = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t warps_needed = n_hist;
-    const int64_t blocks = std::min<int64_t>((warps_needed + 7) / 8, int64_t(n_sm) * 8);
-    k_lemma<<<int(blocks), 256, 0, st>>>(n_hist, len, l, s, x, out);
+    const size_t smem = size_t(2) * len * sizeof(double);
+    if (smem > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(k_lemma, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (e != cudaSuccess) return e;
+    }
+    k_lemma<<<(n_hist + 255) / 256, 256, smem, st>>>(n_hist, len, l, s, x, out);
     return cudaGetLastError();
 }
 

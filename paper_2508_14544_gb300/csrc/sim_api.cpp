@@ -471,8 +471,8 @@ void sim_destroy(sim_ctx *c) {
 
 int sim_cr_amin_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *cr_out,
                       int device_ptrs, void *cuda_stream) {
-    if (n_hist < 0 || len < 1 || l < 1 || !(s >= 0.0) || int64_t(l) + len - 1 > INT32_MAX)
-        return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_lemma: need n_hist >= 0, len >= 1, l >= 1, s >= 0");
+    if (n_hist < 0 || len < 1 || len > 8192 || l < 1 || !(s >= 0.0) || int64_t(l) + len - 1 > INT32_MAX)
+        return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_lemma: need n_hist >= 0, 1 <= len <= 8192, l >= 1, s >= 0");
     if (n_hist == 0) return SIM_OK;
     if (!x || !cr_out) return fail(nullptr, SIM_E_INVAL, "sim_cr_amin_lemma: NULL x or cr_out");
     cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
