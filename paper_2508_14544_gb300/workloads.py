@@ -32,6 +32,11 @@ import numpy as np
 
 __all__ = [
     "Workload",
+    "lookalike_pool",
+    "intervals_rough",
+    "intervals_buckets",
+    "intervals_overlap",
+    "make_sweep",
     "WORKLOADS",
     "make_workload",
     "make_instance",
@@ -261,3 +266,86 @@ def make_workload(name: str, instances: Sequence[int] | range | None = None) -> 
     w = concat_instances(name, spec.M, parts, [p["alpha"] for p in parts], ids)
     w.seed0 = spec.seed0
     return w
+
+
+# --- the paper's experiment setups (Section 6) on a synthetic stand-in for its dataset ---------
+#
+# The paper samples 2,000 LMSYS-Chat-1M conversations and prints only summary statistics of them
+# (Section 6, "Dataset Overview"): prompt sizes 1..468 (mean 41, median 11, variance 4961), output
+# lengths 1..883 (mean 85, median 43, variance 9702).  The dataset is not available here and none
+# of its items is reproduced: the pool below draws from lognormal distributions truncated to those
+# ranges (rounded to integers, out-of-range draws rejected), with (mu, sigma) fitted to the printed
+# mean, median and variance.  Fitted: prompts mu 2.3505, sigma 2.0308 (mean 39.8, median 11,
+# variance 5033); outputs mu 3.8006, sigma 1.1094 (mean 78.3, median 44, variance 9903).
+
+_LOOKALIKE_S = (2.3505, 2.0308, 1, 468)
+_LOOKALIKE_O = (3.8006, 1.1094, 1, 883)
+SWEEP_SEED0 = 5_000_000
+
+
+def _trunc_lognormal(rng: np.random.Generator, n: int, mu: float, sigma: float, lo: int, hi: int) -> np.ndarray:
+    out = np.empty(0, dtype=np.int64)
+    while out.size < n:
+        v = np.rint(np.exp(rng.normal(mu, sigma, size=2 * (n - out.size) + 16))).astype(np.int64)
+        out = np.concatenate([out, v[(v >= lo) & (v <= hi)]])
+    return out[:n]
+
+
+def lookalike_pool(seed: int, n: int = 2000) -> tuple[np.ndarray, np.ndarray]:
+    """(s, o) of a pool of n synthetic requests shaped like the paper's sample."""
+    rng = np.random.default_rng([SWEEP_SEED0, seed])
+    s = _trunc_lognormal(rng, n, *_LOOKALIKE_S)
+    o = _trunc_lognormal(rng, n, *_LOOKALIKE_O)
+    return s, o
+
+
+def intervals_rough(o: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """Experiment 1 (rough prediction): [1, 1000] for every request."""
+    return np.ones_like(o), np.full_like(o, 1000)
+
+
+def intervals_buckets(o: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """Experiment 2 (non-overlapping classification): the bucket [100b + 1, 100b + 100] holding o."""
+    l = 100 * ((o - 1) // 100) + 1
+    return l, l + 99
+
+
+def intervals_overlap(o: np.ndarray, x: Fraction) -> tuple[np.ndarray, np.ndarray]:
+    """Experiment 3 (overlapping intervals): [(1 - x) o, (1 + x) o] with the ends rounded outwards
+    (floor, ceil) in exact integer arithmetic and l >= 1, so l <= o <= u."""
+    a, b = x.numerator, x.denominator
+    o64 = o.astype(np.int64)
+    l = np.maximum(((b - a) * o64) // b, 1)
+    u = -((-(b + a) * o64) // b)
+    return l, u
+
+
+def make_sweep(experiment: str, loads: Sequence[int] = tuple(range(200, 2001, 200)), seeds: int = 4,
+               M: int = 10000) -> Workload:
+    """Instances of the paper's load sweep (Section 6, "Experiment Setup"): for each seed a pool
+    of 2000 requests, and for each load n a random subset of n of them, all arriving at t = 0, with
+    the intervals of ``experiment``: "rough", "buckets" or "overlap:a/b" (x = a/b).  Instance
+    order: seed-major, then load.  ``instance_ids`` holds (seed, n) pairs encoded as
+    seed * 100000 + n."""
+    if experiment == "rough":
+        fn = intervals_rough
+    elif experiment == "buckets":
+        fn = intervals_buckets
+    elif experiment.startswith("overlap:"):
+        x = Fraction(experiment.split(":", 1)[1])
+        if not 0 < x < 1:
+            raise ValueError("overlap x must lie in (0, 1)")
+        fn = lambda o: intervals_overlap(o, x)  # noqa: E731
+    else:
+        raise ValueError(f"unknown experiment {experiment!r}")
+    parts, ids = [], []
+    for seed in range(seeds):
+        s_pool, o_pool = lookalike_pool(seed)
+        rng = np.random.default_rng([SWEEP_SEED0, seed, 1])
+        for n in loads:
+            pick = rng.choice(s_pool.size, size=int(n), replace=False)
+            s, o = s_pool[pick], o_pool[pick]
+            l, u = fn(o)
+            parts.append(dict(a=np.zeros(int(n), np.int32), s=s, o=o, l=l, u=u))
+            ids.append(seed * 100000 + int(n))
+    return concat_instances(f"sweep-{experiment}", M, parts, None, np.asarray(ids, np.int64))

@@ -96,3 +96,14 @@ def test_noalloc_rejects_new_policies():
         rc = lib().sim_run_noalloc(pol, w.M, 1, w.offsets.ctypes.data, None, None, None, None, None,
                                    res.ctypes.data, None)
         assert rc == -1
+
+
+@pytest.mark.parametrize("experiment", ["rough", "buckets", "overlap:1/10", "overlap:99/100"])
+def test_sweep_instances_match_oracle(experiment):
+    """The paper's experiment setups (Section 6) on the dataset stand-in: one seed, loads
+    200..2000, every policy, bit-exact against the oracle."""
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_sweep(experiment, seeds=1)
+    for pol in (0, 1, 2, 4):
+        got, _ = gpu_run(pol, w)
+        assert_same(got, oracle_run(pol, w), tag=f"{experiment} pol={pol}")
