@@ -44,67 +44,11 @@ __device__ T block_reduce(T v, T *sh, bool is_max) {
     return acc;
 }
 
-__global__ void __launch_bounds__(256) k_stage(StageParams S) {
-    __shared__ int64_t sh64[32];
-    const int inst = blockIdx.x;
-    const int64_t base = S.off[inst];
-    const int n = int(S.off[inst + 1] - base);
-    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, work = 0;
-    for (int j = threadIdx.x; j < n; j += blockDim.x) {
-        const int64_t g = base + j;
-        const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
-        if (s < 1 || a < 0 || l < 1 || l > o || o > u) bad_inval = 1;
-        if (int64_t(s) + o > S.M) bad_inf = 1;
-        if ((S.policy == P_AMAX || S.policy == P_AELL) && int64_t(s) + u > S.M) bad_inf = 1;
-        int key;
-        switch (S.policy) {
-            case P_AMAX: key = u; break;
-            case P_HSF: key = o; break;
-            case P_AR: key = S.rank[g]; break;
-            case P_AELL: key = 2 * min(a, kAellMaxStep); break;
-            default: key = l; break;
-        }
-        if (S.policy == P_AR && key < 0) bad_inval = 1;
-        if (S.policy == P_AELL) {
-            if (a > kAellMaxStep) bad_inval = 1;
-            S.lu[g] = make_int2(l, u);  // indexed by request: j == idx below
-        }
-        QEnt e;
-        e.key = key;
-        e.idx = j;
-        e.s = s;
-        e.o = o;
-        S.rec[g] = e;
-        S.rec_a[g] = a;
-        sum_a += a;
-        sum_o += o;
-        work += int64_t(s) * o + int64_t(o) * o / 2;
-    }
-    bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
-    bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
-    sum_a = block_reduce<int64_t>(sum_a, sh64, false);
-    sum_o = block_reduce<int64_t>(sum_o, sh64, false);
-    work = block_reduce<int64_t>(work, sh64, false);
-    int status = ST_OK;
-    if (bad_inval) status = ST_INVAL;
-    else if (bad_inf) status = ST_INFEASIBLE;
-    if (threadIdx.x == 0) {
-        InstInfo in;
-        in.base = base;
-        in.n = n;
-        in.status = status;
-        in.sum_a = sum_a;
-        in.cap = S.step_cap > 0 ? S.step_cap : 64 * (int64_t(n) + sum_o);
-        in.work = work;
-        S.info[inst] = in;
-    }
-    if (status != ST_OK || n <= 1) return;
-    __syncthreads();
-    // bitonic sort of [base, base + n) by (a, key, idx), padded virtually to a power of two
+// Bitonic sort of n records by (a, key, idx) in place, padded virtually to a power of two
+// (positions >= n take no part).  R/RA are shared or global memory.
+__device__ void bitonic_sort(QEnt *R, int32_t *RA, int n) {
     int N = 1;
     while (N < n) N <<= 1;
-    QEnt *R = S.rec + base;
-    int32_t *RA = S.rec_a + base;
     for (int k = 2; k <= N; k <<= 1) {
         for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
             const int half = k >> 1;
@@ -142,6 +86,79 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
     }
 }
 
+// Instances of up to this many requests are sorted in shared memory (20 bytes per request).
+constexpr int kStageSmemN = 2048;
+
+__global__ void __launch_bounds__(256) k_stage(StageParams S) {
+    __shared__ int64_t sh64[32];
+    extern __shared__ __align__(16) unsigned char stage_smem[];
+    const int inst = blockIdx.x;
+    const int64_t base = S.off[inst];
+    const int n = int(S.off[inst + 1] - base);
+    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, work = 0;
+    const bool in_smem = n <= kStageSmemN;
+    QEnt *R = in_smem ? reinterpret_cast<QEnt *>(stage_smem) : S.rec + base;
+    int32_t *RA = in_smem ? reinterpret_cast<int32_t *>(stage_smem + size_t(kStageSmemN) * sizeof(QEnt))
+                          : S.rec_a + base;
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+        const int64_t g = base + j;
+        const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
+        if (s < 1 || a < 0 || l < 1 || l > o || o > u) bad_inval = 1;
+        if (int64_t(s) + o > S.M) bad_inf = 1;
+        if ((S.policy == P_AMAX || S.policy == P_AELL) && int64_t(s) + u > S.M) bad_inf = 1;
+        int key;
+        switch (S.policy) {
+            case P_AMAX: key = u; break;
+            case P_HSF: key = o; break;
+            case P_AR: key = S.rank[g]; break;
+            case P_AELL: key = 2 * min(a, kAellMaxStep); break;
+            default: key = l; break;
+        }
+        if (S.policy == P_AR && key < 0) bad_inval = 1;
+        if (S.policy == P_AELL) {
+            if (a > kAellMaxStep) bad_inval = 1;
+            S.lu[g] = make_int2(l, u);  // indexed by request: j == idx below
+        }
+        QEnt e;
+        e.key = key;
+        e.idx = j;
+        e.s = s;
+        e.o = o;
+        R[j] = e;
+        RA[j] = a;
+        sum_a += a;
+        sum_o += o;
+        work += int64_t(s) * o + int64_t(o) * o / 2;
+    }
+    bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
+    bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
+    sum_a = block_reduce<int64_t>(sum_a, sh64, false);
+    sum_o = block_reduce<int64_t>(sum_o, sh64, false);
+    work = block_reduce<int64_t>(work, sh64, false);
+    int status = ST_OK;
+    if (bad_inval) status = ST_INVAL;
+    else if (bad_inf) status = ST_INFEASIBLE;
+    if (threadIdx.x == 0) {
+        InstInfo in;
+        in.base = base;
+        in.n = n;
+        in.status = status;
+        in.sum_a = sum_a;
+        in.cap = S.step_cap > 0 ? S.step_cap : 64 * (int64_t(n) + sum_o);
+        in.work = work;
+        S.info[inst] = in;
+    }
+    __syncthreads();
+    if (status == ST_OK && n > 1) bitonic_sort(R, RA, n);
+    if (in_smem) {
+        // write the (sorted, or for a rejected instance unsorted) records out
+        for (int j = threadIdx.x; j < n; j += blockDim.x) {
+            S.rec[base + j] = R[j];
+            S.rec_a[base + j] = RA[j];
+        }
+    }
+}
+
 __global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= n) return;
@@ -156,7 +173,8 @@ __global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out,
 
 cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
     if (p.n_inst <= 0) return cudaSuccess;
-    k_stage<<<p.n_inst, 256, 0, st>>>(p);
+    const size_t smem = size_t(kStageSmemN) * (sizeof(QEnt) + sizeof(int32_t));  // 40 KB
+    k_stage<<<p.n_inst, 256, smem, st>>>(p);
     return cudaGetLastError();
 }
 
