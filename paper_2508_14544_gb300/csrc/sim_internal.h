@@ -30,6 +30,8 @@ struct InstInfo {
     int64_t work;     // cost estimate used to order instances (longest first)
     int32_t n;        // number of requests
     int32_t status;   // 0 or a sim_status from validation
+    int32_t lmax;     // largest u_i or o_i of the instance (bounds every projected length)
+    int32_t pad;
 };
 
 struct DevResult {

@@ -41,6 +41,7 @@
 // M, and the admitted count is the minimum of those, less one.
 #include <climits>
 #include <cstdint>
+#include <type_traits>
 
 #include "sim_internal.h"
 
@@ -75,7 +76,20 @@ __device__ __forceinline__ QEnt proj(const RunParams &P, int64_t base, QEnt e) {
     return e;
 }
 
-__device__ __forceinline__ int sat32(int64_t v) {
+// Memory sums of the active set (projected memory at an endpoint, the next step's memory) are
+// compared with M <= 2^26.  The shared-memory kernel computes them in 32 bits: every instance it
+// runs has capacity x (2 lmax + 2) + 2^27 < 2^31 (lmax = the longest u or o of the instance), and
+// then every offset from the time base (E - tb, y - tb, t - tb) is at most lmax + 1 in size, every
+// product (count x offset) at most capacity x (lmax + 1), and every sum of B + tb at most the
+// memory of a step, so nothing overflows.  Instances outside that bound, and instances whose set
+// outgrows shared memory, run in the global-memory kernel, which keeps 64 bits and saturates at
+// 2^30 (enough for every comparison with M).
+template <bool N>
+using wint = typename std::conditional<N, int32_t, int64_t>::type;
+
+template <bool N>
+__device__ __forceinline__ int satw(wint<N> v) {
+    if (N) return int(v);
     const int64_t hi = int64_t(1) << 30;
     return int(v > hi ? hi : (v < -hi ? -hi : v));
 }
@@ -410,6 +424,7 @@ __device__ __forceinline__ void store_job(const Ws &w, int i, int e, int f, int 
 }
 
 // SB, PM, SB0 and min F for the A entries (no dead entries), time base tb.
+template <bool N>
 __device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int &nextF) {
     const int lane = lane_id();
     int carry = 0;
@@ -452,8 +467,8 @@ __device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int
         for (int j = 0; j < 4; ++j) {
             int h = INT_MIN;
             if (base + j < A) {
-                const int64_t e = int64_t(ee[j]) - tb;
-                h = sat32(int64_t(ss[j]) + int64_t(A - base - j) * e + e);
+                const wint<N> e = wint<N>(ee[j]) - tb;
+                h = satw<N>(wint<N>(ss[j]) + wint<N>(A - base - j) * e + e);
                 fmin = min(fmin, ff[j]);
             }
             mx = max(mx, h);
@@ -503,10 +518,11 @@ __device__ __forceinline__ void compact(const Ws &w, int &A) {
 // Remove the entries marked dead (F < 0) and recompute the derived arrays, in one pass when the
 // set fits one chunk (positions, suffix sums and prefix maxima of the compacted order are known
 // from the live counts before anything is stored).
+template <bool N>
 __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int &SB0, int &nextF) {
     if (A > kChunk) {
         compact(w, A);
-        derive(w, A, tb, SB0, nextF);
+        derive<N>(w, A, tb, SB0, nextF);
         return;
     }
     const int lane = lane_id();
@@ -540,8 +556,8 @@ __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int 
     for (int j = 0; j < 4; ++j) {
         qp[j] = q;
         if (lv[j]) {
-            const int64_t e = int64_t(ee[j]) - tb;
-            mx = max(mx, sat32(int64_t(sfx[j] + after) + int64_t(L - q) * e + e));
+            const wint<N> e = wint<N>(ee[j]) - tb;
+            mx = max(mx, satw<N>(wint<N>(sfx[j] + after) + wint<N>(L - q) * e + e));
             fmin = min(fmin, ff[j]);
             ++q;
         }
@@ -606,6 +622,7 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
 // Largest admissible prefix of the window at step t (see the file comment), for any active-set
 // size: per point a binary search for the first failing prefix length.  Lane m holds window entry
 // m (m < W); the active set is compact with derived arrays for time base tb.
+template <bool N>
 __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int tb, int SB0, int64_t M, int t,
                                                         int W, const QEnt &mine) {
     const int lane = lane_id();
@@ -620,46 +637,46 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
     }
     if (lane == 0) w.wcs[0] = 0;
     __syncwarp();
-    const int64_t dt = int64_t(t) - tb;
-    const int64_t need = int64_t(SB0) + int64_t(A) * dt;
-    const int64_t csW = tot;
+    const wint<N> dt = wint<N>(t) - tb;
+    const wint<N> need = wint<N>(SB0) + wint<N>(A) * dt;
+    const wint<N> csW = tot;
     // the coming step (x = t): every window entry adds s + 1
-    const unsigned ball = __ballot_sync(FULL, lane < W && need + incl > M);
+    const unsigned ball = __ballot_sync(FULL, lane < W && need + incl > wint<N>(M));
     int phi = ball ? __ffs(ball) : W + 1;
     // active endpoints x = E_j >= t
     for (int j = lane; j < A; j += 32) {
         const int ej = w.E[j];
         if (ej < t) continue;
-        const int64_t d = int64_t(ej) - t;
-        const int64_t v0 = int64_t(w.SB[j]) + int64_t(A - j) * (int64_t(ej) - tb);
-        if (v0 + csW + int64_t(W) * d <= M) continue;
-        if (v0 > M) {
+        const wint<N> d = wint<N>(ej) - t;
+        const wint<N> v0 = wint<N>(w.SB[j]) + wint<N>(A - j) * (wint<N>(ej) - tb);
+        if (v0 + csW + wint<N>(W) * d <= wint<N>(M)) continue;
+        if (v0 > wint<N>(M)) {
             phi = 0;
             continue;
         }
-        const int r = lane_prefix_count(W, [&](int m) { return int64_t(w.wkey[m]) <= d; });
+        const int r = lane_prefix_count(W, [&](int m) { return wint<N>(w.wkey[m]) <= d; });
         if (r >= W) continue;
-        const int64_t base = v0 - w.wcs[r] - int64_t(r) * d;
-        if (base + csW + int64_t(W) * d <= M) continue;
+        const wint<N> base = v0 - w.wcs[r] - wint<N>(r) * d;
+        if (base + csW + wint<N>(W) * d <= wint<N>(M)) continue;
         int lo = r + 1, hi = W;
         while (lo < hi) {
             const int mid = (lo + hi) >> 1;
-            if (base + w.wcs[mid] + int64_t(mid) * d > M) hi = mid; else lo = mid + 1;
+            if (base + w.wcs[mid] + wint<N>(mid) * d > wint<N>(M)) hi = mid; else lo = mid + 1;
         }
         phi = min(phi, lo);
     }
     // the window entries' own last steps x = t + key_m - 1
     if (lane < W) {
-        const int64_t d = int64_t(mine.key) - 1;
-        const int64_t y = int64_t(t) + d;
-        const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
-        const int64_t av = int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb);
-        const int64_t base = av - ex - int64_t(lane) * d;  // ex = CS[lane]
-        if (base + csW + int64_t(W) * d > M) {
+        const wint<N> d = wint<N>(mine.key) - 1;
+        const wint<N> y = wint<N>(t) + d;
+        const int lb = lane_prefix_count(A, [&](int i) { return wint<N>(w.E[i]) < y; });
+        const wint<N> av = wint<N>(w.SB[lb]) + wint<N>(A - lb) * (y - tb);
+        const wint<N> base = av - ex - wint<N>(lane) * d;  // ex = CS[lane]
+        if (base + csW + wint<N>(W) * d > wint<N>(M)) {
             int lo = lane + 1, hi = W;
             while (lo < hi) {
                 const int mid = (lo + hi) >> 1;
-                if (base + w.wcs[mid] + int64_t(mid) * d > M) hi = mid; else lo = mid + 1;
+                if (base + w.wcs[mid] + wint<N>(mid) * d > wint<N>(M)) hi = mid; else lo = mid + 1;
             }
             phi = min(phi, lo);
         }
@@ -673,9 +690,10 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
 // (candidate k-1 adds s + 1 + (x - t) at every point x it reaches: the coming step x = t, the
 // active endpoints E_j with key > E_j - t, and the endpoints of window entries 0..k-1); the first
 // k at which any point exceeds M ends the prefix.  Falls back to the binary-search form otherwise.
+template <bool N>
 __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int W,
                                                  const QEnt &mine) {
-    if (A > kChunk) return admissible_prefix_search(w, A, tb, SB0, M, t, W, mine);
+    if (A > kChunk) return admissible_prefix_search<N>(w, A, tb, SB0, M, t, W, mine);
     const int lane = lane_id();
     const int Mi = int(M);
     // active endpoints at or after t: V(E_j) and d_j = E_j - t
@@ -688,7 +706,7 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     for (int j = 0; j < 4; ++j) {
         const bool ok = base + j < A && ee[j] >= t;
         da[j] = ok ? ee[j] - t : INT_MAX;
-        va[j] = ok ? sat32(int64_t(ss[j]) + int64_t(A - base - j) * (int64_t(ee[j]) - tb)) : INT_MIN;
+        va[j] = ok ? satw<N>(wint<N>(ss[j]) + wint<N>(A - base - j) * (wint<N>(ee[j]) - tb)) : INT_MIN;
     }
     // this lane's window entry: V(y) of the active set at its last step y = t + key - 1
     const int dm = mine.key - 1;
@@ -697,9 +715,9 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     if (lane < W) {
         const int64_t y = int64_t(t) + dm;
         const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
-        av = sat32(int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb));
+        av = satw<N>(wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb));
     }
-    int64_t need = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
+    wint<N> need = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
     // two candidates per round: the state after both is used only if neither fails
     for (int k = 1; k <= W; k += 2) {
         const bool two = k < W;
@@ -707,8 +725,8 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
         const int k1 = __shfl_sync(FULL, mine.key, k - 1);
         const int s2 = __shfl_sync(FULL, mine.s, k) + 1;
         const int k2 = __shfl_sync(FULL, mine.key, k);
-        const int64_t need1 = need + s1;
-        const int64_t need2 = need1 + s2;
+        const wint<N> need1 = need + s1;
+        const wint<N> need2 = need1 + s2;
         bool f1 = false, f2 = false;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -725,9 +743,9 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
         f2 = f2 || vc > Mi;
         const unsigned b1 = __ballot_sync(FULL, f1);
         const unsigned b2 = __ballot_sync(FULL, f2);
-        if (b1 != 0 || need1 > M) return k - 1;
+        if (b1 != 0 || need1 > wint<N>(M)) return k - 1;
         if (!two) break;
-        if (b2 != 0 || need2 > M) return k;
+        if (b2 != 0 || need2 > wint<N>(M)) return k;
         need = need2;
     }
     return W;
@@ -739,22 +757,23 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
 // in the K array (these policies do not use it) and each window entry m accumulates, in a register,
 // the candidates so far whose length is >= L_m (itself included); entry m's point counts once m is
 // admitted.  Any active-set size.
+template <bool N>
 __device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int tb, int SB0, int64_t M, int t,
                                                          int W, const QEnt &mine) {
     const int lane = lane_id();
     const int Mi = int(M);
     for (int j = lane; j < A; j += 32) {
         const int ej = w.E[j];
-        w.K[j] = (ej >= t) ? sat32(int64_t(w.SB[j]) + int64_t(A - j) * (int64_t(ej) - tb)) : INT_MIN;
+        w.K[j] = (ej >= t) ? satw<N>(wint<N>(w.SB[j]) + wint<N>(A - j) * (wint<N>(ej) - tb)) : INT_MIN;
     }
     const int Lm = mine.key, dm = Lm - 1;
     int av = 0, acc = 0;
     if (lane < W) {
         const int64_t y = int64_t(t) + dm;
         const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
-        av = sat32(int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb));
+        av = satw<N>(wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb));
     }
-    int64_t need = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
+    wint<N> need = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
     for (int k = 1; k <= W; ++k) {
         const int c = k - 1;
         const int sc = __shfl_sync(FULL, mine.s, c) + 1;
@@ -771,8 +790,8 @@ __device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int
             }
         }
         if (lane < W && Lc >= Lm) acc += sc + dm;
-        if (lane <= c) fail = fail || int64_t(av) + acc > M;
-        if (__ballot_sync(FULL, fail) != 0 || need > M) return k - 1;
+        if (lane <= c) fail = fail || wint<N>(av) + acc > wint<N>(M);
+        if (__ballot_sync(FULL, fail) != 0 || need > wint<N>(M)) return k - 1;
     }
     return W;
 }
@@ -838,7 +857,7 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
 // ---------------------------------------------------------------------------------------------
 // One instance, simulated by one warp.  All lanes hold identical copies of the scalar state.
 // ---------------------------------------------------------------------------------------------
-template <int POL>
+template <int POL, bool N>
 __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
     const int lane = lane_id();
     const InstInfo info = P.info[inst];
@@ -847,6 +866,11 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
     r.status = info.status;
     r.pad = 0;
     if (info.status != ST_OK || info.n == 0) {
+        if (lane == 0) P.res[inst] = r;
+        return;
+    }
+    if (N && int64_t(P.ca) * (2 * int64_t(info.lmax) + 2) + (int64_t(1) << 27) >= (int64_t(1) << 31)) {
+        r.status = kStatusCapacity;  // too long for 32-bit sums: the global-memory kernel runs it
         if (lane == 0) P.res[inst] = r;
         return;
     }
@@ -891,7 +915,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             // removal share this one site: the loop body stays small, which matters when two
             // warps at different points of it share a scheduler's instruction cache.
             tb = tb_next;
-            compact_derive(w, A, tb, SB0, nextF);
+            compact_derive<N>(w, A, tb, SB0, nextF);
             pend_compact = false;
             pdirty = true;
         }
@@ -924,9 +948,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
         }
         // ---- S2/S3: A_min overflow of the next step -> cancel in ascending (estimate, index)
         if (POL == P_AMIN) {
-            int64_t need = int64_t(SB0) + int64_t(A) * (t - tb);
-            if (need > M) {
-                while (need > M) {
+            wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
+            if (need > wint<N>(M)) {
+                while (need > wint<N>(M)) {
                     unsigned bk = UINT_MAX, bi = UINT_MAX;
                     int bp = -1;
                     for (int cb = 0; cb < A; cb += kChunk) {
@@ -963,7 +987,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                     __syncwarp();
                     if (lane == 0) w.F[pos] = -1;
                     __syncwarp();
-                    need -= int64_t(b) + t;
+                    need -= wint<N>(b) + t;
                     ++nev;
                     delta_insert(w, q, e);
                 }
@@ -1009,9 +1033,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 pdirty = true;
             }
             // quick test of the head alone (the prefix of length one)
-            const int64_t dt = int64_t(t) - tb;
-            const int64_t need = int64_t(SB0) + int64_t(A) * dt;
-            bool fits = need + h.s + 1 <= M;
+            const wint<N> dt = wint<N>(t) - tb;
+            const wint<N> need = wint<N>(SB0) + wint<N>(A) * dt;
+            bool fits = need + h.s + 1 <= wint<N>(M);
             if (fits && A > 0) {
                 const int64_t y = int64_t(t) + h.key - 1;
                 if (pdirty || y != y_prev + 1) {
@@ -1023,9 +1047,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 }
                 pdirty = false;
                 y_prev = y;
-                if (int64_t(w.PM[hi]) + h.s + 1 - dt > M) fits = false;
-                const int64_t v = int64_t(w.SB[lb]) + int64_t(A - lb) * (y - tb);
-                if (v + h.s + h.key > M) fits = false;
+                // PM[0] is the INT_MIN sentinel: compare without adding to it
+                if (wint<N>(w.PM[hi]) > wint<N>(M) - h.s - 1 + dt) fits = false;
+                const wint<N> v = wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb);
+                if (v + h.s + h.key > wint<N>(M)) fits = false;
             } else if (fits) {
                 fits = int64_t(h.s) + h.key <= M;
             }
@@ -1039,8 +1064,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 if (lane < W) mine = proj<POL>(P, info.base, mine);
             }
             const int Kadm = (POL == P_AR || POL == P_AELL)
-                                 ? admissible_prefix_general(w, A, tb, SB0, M, t, W, mine)
-                                 : admissible_prefix(w, A, tb, SB0, M, t, W, mine);
+                                 ? admissible_prefix_general<N>(w, A, tb, SB0, M, t, W, mine)
+                                 : admissible_prefix<N>(w, A, tb, SB0, M, t, W, mine);
             if (Kadm <= 0) {
                 status = ST_STATE;  // the head test and the window disagree: internal error
                 break;
@@ -1055,7 +1080,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 break;
             }
             tb = t;
-            derive(w, A, tb, SB0, nextF);
+            derive<N>(w, A, tb, SB0, nextF);
             pdirty = true;
             if (Kadm < W) {
                 // window entry Kadm is the new head, and it does not fit at step t
@@ -1071,8 +1096,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
         if (status != ST_OK) break;
         // ---- S6: process the batch
         if (t == nextF) {
-            const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) - tb);
-            if (mem > M) {
+            const wint<N> mem = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
+            if (mem > wint<N>(M)) {
                 status = ST_STATE;
                 break;
             }
@@ -1149,7 +1174,7 @@ __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
         k = __shfl_sync(FULL, k, 0);
         if (k >= P.n_work) break;
         const int inst = P.work ? P.work[k] : k;
-        sim_instance<POL>(P, w, inst);
+        sim_instance<POL, SMEM>(P, w, inst);
     }
 }
 

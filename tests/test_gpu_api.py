@@ -165,3 +165,29 @@ def test_unsorted_arrivals():
         ref, rcomp = oracle_run(pol, w, completions=True)
         assert_same(got, ref, tag="unsorted")
         assert np.array_equal(comp, rcomp)
+
+
+def test_long_requests_narrow_and_wide_kernels_agree():
+    """Lengths of ~3e5 steps: with the default 512-slot shared-memory capacity the 32-bit kernel is
+    valid (512 x (2 lmax + 2) + 2^27 < 2^31); with a 4096-slot capacity it is not, so every
+    instance is re-run by the 64-bit global-memory kernel.  Both equal the oracle."""
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(21)
+    parts = []
+    M = 1_000_000
+    for _ in range(6):
+        n = 12
+        o = rng.integers(1000, 300_000, n)
+        l = np.maximum(o // 3, 1)
+        u = np.minimum(o * 2, M - 100)
+        s = rng.integers(1, 50, n)
+        a = rng.integers(0, 200_000, n)
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    w = W.concat_instances("long", M, parts)
+    for pol in (0, 1, 2, 4):
+        ref = oracle_run(pol, w)
+        narrow, _ = gpu_run(pol, w)
+        wide, _ = gpu_run(pol, w, smem_active_cap=4096)
+        for f in FIELDS:
+            assert np.array_equal(narrow[f], ref[f]), (pol, f)
+            assert np.array_equal(wide[f], ref[f]), (pol, f)
