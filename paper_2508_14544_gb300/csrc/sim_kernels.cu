@@ -824,34 +824,38 @@ __device__ __forceinline__ void sort_admitted(const Ws &w, int K, QEnt &mine) {
 // group at y = E[j] (whose prefix maximum is PM[j+1]: within a group of equal E that lies at or
 // after tb the first entry has the largest H).  Conditions (1)-(3) give, per interval, a lower
 // bound on y from (2) and upper bounds from (1) and (3).
+// All quantities are taken relative to the time base tb (they stay within the 32-bit bound of the
+// shared-memory kernel); PM[0] is the -infinity sentinel and takes no arithmetic.
+template <bool N>
 __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int s,
                                                   int L, int64_t tau_lim) {
+    using W = wint<N>;
     const int lane = lane_id();
-    const int64_t y0 = int64_t(t) + L - 1;
-    const int64_t ylim = tau_lim - 1 + L - 1;
-    const int64_t tau1 = tb + floor_div32(M - s - 1 - SB0, A);  // (1)
-    const int64_t yup = min(ylim, tau1 + L - 1);
+    const W BIG = N ? W(1 << 29) : W(int64_t(1) << 60);
+    const W y0 = W(t - tb) + L - 1;
+    const W ylim = W(min(tau_lim - tb, int64_t(BIG))) - 1 + L - 1;
+    const W tau1 = floor_div32(M - s - 1 - SB0, A);  // (1)
+    const W yup = min(ylim, tau1 + L - 1);
     if (yup <= y0) return kBig;
-    const int64_t C2 = M - s - L - tb;
-    const int64_t C3 = M - s - L;
-    int64_t best = kBig;
+    const W C = W(M) - s - L;  // (2): PM - C <= y;  (3): y <= floor((C - SB[j]) / (A - j))
+    W best = BIG;
     for (int j = lane; j <= A; j += 32) {
-        const int64_t prev = (j == 0) ? -kBig : int64_t(w.E[j - 1]);
-        const int64_t cur = (j == A) ? kBig : int64_t(w.E[j]);
+        const W prev = (j == 0) ? -BIG : W(w.E[j - 1] - tb);
+        const W cur = (j == A) ? BIG : W(w.E[j] - tb);
         if (cur <= y0 || prev >= yup) continue;
-        const int64_t y3 = (A - j > 0) ? tb + floor_div32(C3 - w.SB[j], A - j) : kBig;
-        const int64_t up = min(yup, y3);
-        const int64_t lo = max(prev + 1, y0 + 1);
-        const int64_t cand = max(lo, int64_t(w.PM[j]) - C2);
+        const W y3 = (A - j > 0) ? W(floor_div32(int64_t(C) - w.SB[j], A - j)) : BIG;
+        const W up = min(yup, y3);
+        const W lo = max(prev + 1, y0 + 1);
+        const W cand = (j == 0) ? lo : max(lo, W(w.PM[j]) - C);
         if (cand <= min(cur - 1, up)) best = min(best, cand);
-        if (j < A && cur > prev && cur >= y0 + 1 && cur <= up && int64_t(w.PM[j + 1]) - C2 <= cur)
+        if (j < A && cur > prev && cur >= y0 + 1 && cur <= up && W(w.PM[j + 1]) - C <= cur)
             best = min(best, cur);
     }
-    // warp minimum: candidates lie in (y0, yup] and steps fit 31 bits, so y - y0 fits 32 bits
-    const unsigned off = (best == kBig) ? UINT_MAX : unsigned(best - y0);
+    // warp minimum: candidates lie in (y0, yup], so y - y0 fits 32 bits
+    const unsigned off = (best == BIG) ? UINT_MAX : unsigned(best - y0);
     const unsigned m = __reduce_min_sync(FULL, off);
     if (m == UINT_MAX) return kBig;
-    return y0 + m - L + 1;
+    return int64_t(tb) + int64_t(y0) + m - L + 1;
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -1130,7 +1134,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             if (POL == P_AELL && A > 0) tau = min(tau, int64_t(w.E[0]) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
             if (tau > int64_t(t) + 1 && hvalid && A > 0)
-                tau = min(tau, first_fit_step(w, A, tb, SB0, M, t, h.s, h.key, tau));
+                tau = min(tau, first_fit_step<N>(w, A, tb, SB0, M, t, h.s, h.key, tau));
             const int64_t c = max(tau - int64_t(t), int64_t(1));
             const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) + c - 1 - tb);
             if (mem > M) {
