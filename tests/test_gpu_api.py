@@ -191,3 +191,19 @@ def test_long_requests_narrow_and_wide_kernels_agree():
         for f in FIELDS:
             assert np.array_equal(narrow[f], ref[f]), (pol, f)
             assert np.array_equal(wide[f], ref[f]), (pol, f)
+
+
+def test_command_lines(capsys):
+    """`python -m paper_2508_14544_gb300.run` and `.sweep` through the C ABI."""
+    import json
+
+    from paper_2508_14544_gb300 import run, sweep
+    run.main(["--workload", "c1", "--policy", "A_ell", "--repeat", "2"])
+    lines = [json.loads(l) for l in capsys.readouterr().out.splitlines() if l.startswith("{")]
+    assert len(lines) == 2 and lines[0]["worst_status"] == 0 and lines[0]["request_steps"] == lines[1]["request_steps"]
+    run.main(["--workload", "c1", "--policy", "A_r"])
+    assert json.loads(capsys.readouterr().out.splitlines()[0])["worst_status"] == 0
+    sweep.main(["--experiments", "buckets", "--policies", "A_min,H-SF", "--seeds", "1"])
+    out = [json.loads(l) for l in capsys.readouterr().out.splitlines() if l.startswith("{")]
+    assert [o["policy"] for o in out] == ["A_min", "H-SF"]
+    assert all(len(o["avg_latency"]) == 10 for o in out)
