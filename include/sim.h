@@ -85,9 +85,15 @@ enum {
                                        memory per instance (default 512).  Instances that need more
                                        are re-run automatically with the active set in global
                                        memory; results are identical. */
-    SIM_OPT_WARPS_PER_SM = 5        /* 0..64: at most this many simulation warps resident per SM
+    SIM_OPT_WARPS_PER_SM = 5,       /* 0..64: at most this many simulation warps resident per SM
                                        (0, the default: as many as shared memory allows).  Results
                                        do not depend on it. */
+    SIM_OPT_DEBUG_CHECKS = 6        /* 0/1: run every instance in the global-memory kernel and check
+                                       the simulation state's invariants between events (active set
+                                       sorted by projected end, suffix sums and prefix maxima of the
+                                       set, queue order; no job past its projected end under A_max,
+                                       H-SF and A_r).  A violation gives that instance SIM_E_STATE.
+                                       Slower; results are otherwise identical. */
 };
 
 /*

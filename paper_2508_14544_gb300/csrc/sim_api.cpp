@@ -29,6 +29,7 @@ struct sim_ctx {
     int record_completions = 0;
     int wpb = 4;
     int warps_per_sm = 0;
+    int debug_checks = 0;
     int smem_ca = 512;
     int dcap = 256;
     // state
@@ -154,6 +155,9 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
         case SIM_OPT_WARPS_PER_SM:
             if (value < 0 || value > 64) return fail(c, SIM_E_INVAL, "WARPS_PER_SM must be in [0, 64]");
             c->warps_per_sm = int(value);
+            return SIM_OK;
+        case SIM_OPT_DEBUG_CHECKS:
+            c->debug_checks = value ? 1 : 0;
             return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
             if (value < 128 || value > 4096 || value % 128)
@@ -335,6 +339,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.ca = ca;
     p.dcap = dcap;
     p.use_smem = smem ? 1 : 0;
+    p.debug = c->debug_checks;
     p.gws = c->d_gws;
     p.gws_stride = int64_t(per_warp);
     p.mainbuf = c->d_main;
@@ -363,7 +368,8 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
             cudaSuccess)
             return cuda_fail(c, e, "cudaMemsetAsync");
     }
-    rc = run_launch(c, st, nullptr, c->n_inst, true);
+    // with SIM_OPT_DEBUG_CHECKS every instance runs in the checking global-memory kernel
+    rc = run_launch(c, st, nullptr, c->n_inst, !c->debug_checks);
     if (rc) return rc;
     c->h_res.resize(size_t(c->n_inst));
     e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost, st);

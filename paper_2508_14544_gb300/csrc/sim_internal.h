@@ -68,6 +68,7 @@ struct RunParams {
     int32_t ca;                // active-set capacity per instance (multiple of 32)
     int32_t dcap;              // delta-queue capacity per instance (multiple of 32)
     int32_t use_smem;          // 1: active set + delta queue in shared memory; 0: global workspace
+    int32_t debug;             // 1: check the simulation state's invariants every iteration (global kernel)
     unsigned char *gws;        // global workspace base (use_smem == 0)
     int64_t gws_stride;        // bytes per warp slot
     QEnt *mainbuf;             // ping-pong main-queue buffers, 2 * main_cap per warp slot

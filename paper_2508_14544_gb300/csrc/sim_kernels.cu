@@ -858,6 +858,37 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
     return int64_t(tb) + int64_t(y0) + m - L + 1;
 }
 
+// Invariants of the simulation state between events (SIM_OPT_DEBUG_CHECKS; global-memory kernel
+// only): the active set is sorted by E; SB and PM are the suffix sums and prefix maxima of the
+// current set and time base; SB0 and nextF match them; under A_max, H-SF and A_r no job runs past
+// its projected last step; the delta queue is strictly descending and the cached head of the main
+// array ascending.  Returns false on the first violation.
+template <int POL, bool N>
+__device__ bool state_ok(const Ws &w, const Queue &q, int A, int tb, int SB0, int nextF) {
+    const int lane = lane_id();
+    bool bad = false;
+    int fmin = INT_MAX;
+    for (int i = lane; i < A; i += 32) {
+        const int e = w.E[i];
+        if (i + 1 < A && e > w.E[i + 1]) bad = true;
+        if (w.SB[i] != w.SB[i + 1] + w.B[i] + tb) bad = true;
+        const wint<N> d = wint<N>(e) - tb;
+        const int h = satw<N>(wint<N>(w.SB[i]) + wint<N>(A - i) * d + d);
+        if (w.PM[i + 1] != max(w.PM[i], h)) bad = true;
+        fmin = min(fmin, w.F[i]);
+        if ((POL == P_AMAX || POL == P_HSF || POL == P_AR) && w.F[i] > e) bad = true;
+    }
+    if (lane == 0 && (w.SB[A] != 0 || w.PM[0] != INT_MIN || (A > 0 && w.SB[0] != SB0))) bad = true;
+    for (int i = lane; i + 1 < q.dn; i += 32)
+        if (!qless(w.dq[i + 1], w.dq[i])) bad = true;
+    if (q.mcb >= 0)
+        for (int i = q.mh + lane; i + 1 < min(q.me, q.mcb + kMc); i += 32)
+            if (i >= q.mcb && !qless(w.mc[i - q.mcb], w.mc[i + 1 - q.mcb])) bad = true;
+    fmin = __reduce_min_sync(FULL, fmin);
+    if (A > 0 && fmin != nextF) bad = true;
+    return __ballot_sync(FULL, bad) == 0;
+}
+
 // ---------------------------------------------------------------------------------------------
 // One instance, simulated by one warp.  All lanes hold identical copies of the scalar state.
 // ---------------------------------------------------------------------------------------------
@@ -922,6 +953,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             compact_derive<N>(w, A, tb, SB0, nextF);
             pend_compact = false;
             pdirty = true;
+        }
+        if (!N && P.debug && !state_ok<POL, N>(w, q, A, tb, SB0, nextF)) {
+            status = ST_STATE;  // a consistency check of SIM_OPT_DEBUG_CHECKS failed
+            break;
         }
         if (steps >= cap) {
             status = ST_STEPCAP;

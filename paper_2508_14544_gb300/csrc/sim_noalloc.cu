@@ -159,6 +159,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
     p.dcap = kNaDeltaCap;
     p.use_smem = 0;
+    p.debug = 0;
     p.gws = base + kOffWs;
     p.gws_stride = int64_t(ws_bytes_max());
     p.mainbuf = reinterpret_cast<simgb::QEnt *>(base + kOffMain);

@@ -207,3 +207,16 @@ def test_command_lines(capsys):
     out = [json.loads(l) for l in capsys.readouterr().out.splitlines() if l.startswith("{")]
     assert [o["policy"] for o in out] == ["A_min", "H-SF"]
     assert all(len(o["avg_latency"]) == 10 for o in out)
+
+
+@pytest.mark.parametrize("pol", [0, 1, 2, 3, 4])
+def test_debug_checks_hold_and_change_nothing(pol):
+    """SIM_OPT_DEBUG_CHECKS: the invariants hold at every event of the 1000-request instances
+    (all alphas) and of an online workload with bursts, and the results are unchanged."""
+    from paper_2508_14544_gb300 import workloads as W
+    for w in (W.make_workload("c2", range(3, 1024, 64)), W.make_workload("c3", [5, 9])):
+        a, _ = gpu_run(pol, w)
+        b, _ = gpu_run(pol, w, debug_checks=1)
+        assert np.all(b["status"] == 0)
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f]), (pol, f)
