@@ -226,6 +226,7 @@ def run_ours(args) -> None:
     # timed region: K steps, device time by CUDA events on the simulator's stream
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    load_starts = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     run_starts = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     run_ends = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     if world > 1:
@@ -239,6 +240,7 @@ def run_ours(args) -> None:
             torch.cuda.synchronize()
             starts[k].record(stream)
             for j, sim in enumerate(sims):
+                load_starts[k][j].record(stream)
                 sim.load(w.offsets, *d_in)
                 run_starts[k][j].record(stream)
                 res[j] = sim.run(sh)
@@ -253,6 +255,7 @@ def run_ours(args) -> None:
     launches = sum(s.kernel_launches() for s in sims) - launches0
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     run_ms = [[run_starts[k][j].elapsed_time(run_ends[k][j]) for j in range(3)] for k in range(args.steps)]
+    load_ms = [[load_starts[k][j].elapsed_time(run_starts[k][j]) for j in range(3)] for k in range(args.steps)]
     total_s = sum(step_ms) / 1000.0
     if world > 1:
         t = torch.tensor([total_s], device=dev, dtype=torch.float64)
@@ -343,6 +346,12 @@ def run_ours(args) -> None:
                    "l2": "256 MB buffer written between timed steps (inputs are 20 MB < L2)",
                    "request_steps_per_step": rs_per_step,
                    "sim_run_ms": dict(zip(POLICY_NAMES, [round(x, 3) for x in per_pol_ms])),
+                   "sim_load_ms": dict(zip(POLICY_NAMES, [round(statistics.mean(load_ms[k][j] for k in range(args.steps)), 3)
+                                                          for j in range(3)])),
+                   "batches_per_s": {POLICY_NAMES[j]: int(res[j]["steps"].sum()) / (per_pol_ms[j] / 1000.0)
+                                     for j in range(3)},
+                   "us_per_instance": {POLICY_NAMES[j]: round(1000.0 * per_pol_ms[j] / w.n_instances, 3)
+                                       for j in range(3)},
                    "further_policies_not_in_step": further,
                    "lemma_evaluator": {"histograms": 1 << 20, "lengths": 64, "ms": round(statistics.median(lm), 4),
                                        "GB_per_s": round(lemma_gbs, 1),
