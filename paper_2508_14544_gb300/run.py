@@ -2,11 +2,13 @@
 
   python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024] [--repeat 1]
 
-Prints one JSON line per run with the wall time of sim_run and totals of the result fields.
+Prints one JSON line per run with the wall time of sim_run, totals of the result fields, the
+throughput and a sha256 of the per-instance result records (equal across runs and launch shapes).
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import time
 
@@ -42,10 +44,14 @@ def main(argv=None) -> None:
             t0 = time.perf_counter()
             res = sim.run()
             dt = time.perf_counter() - t0
+            rs, st = int(res["request_steps"].sum()), int(res["steps"].sum())
+            digest = hashlib.sha256(np.ascontiguousarray(res).tobytes()).hexdigest()
             print(json.dumps({"workload": args.workload, "policy": args.policy, "instances": w.n_instances,
-                              "sim_run_s": dt, "request_steps": int(res["request_steps"].sum()),
-                              "steps": int(res["steps"].sum()), "evictions": int(res["evictions"].sum()),
-                              "worst_status": int(res["status"].min())}), flush=True)
+                              "sim_run_s": dt, "request_steps": rs, "steps": st,
+                              "request_steps_per_s": rs / dt, "steps_per_s": st / dt,
+                              "total_latency": int(res["total_latency"].sum()),
+                              "evictions": int(res["evictions"].sum()),
+                              "worst_status": int(res["status"].min()), "results_sha256": digest}), flush=True)
 
 
 if __name__ == "__main__":
