@@ -410,8 +410,11 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
     c->comp_valid = c->record_completions != 0;
     if (worst == SIM_E_STATE) fail(c, SIM_E_STATE, "sim_run: an internal consistency check failed");
     else if (worst == SIM_E_STEPCAP) fail(c, SIM_E_STEPCAP, "sim_run: an instance hit the step cap");
-    else if (worst == SIM_E_INFEASIBLE) fail(c, SIM_E_INFEASIBLE, "sim_run: an instance has a request with s+o > M (or s+u > M under A_max)");
-    else if (worst == SIM_E_INVAL) fail(c, SIM_E_INVAL, "sim_run: an instance violates 1 <= l <= o <= u, s >= 1, a >= 0");
+    else if (worst == SIM_E_INFEASIBLE)
+        fail(c, SIM_E_INFEASIBLE, "sim_run: an instance has a request with s+o > M (or s+u > M under A_max, A_ell)");
+    else if (worst == SIM_E_INVAL)
+        fail(c, SIM_E_INVAL, "sim_run: an instance violates 1 <= l <= o <= u, s >= 1, a >= 0 (rank >= 0 under A_r, "
+                             "a < 2^30 under A_ell)");
     return worst;
 }
 

@@ -27,7 +27,6 @@ struct InstInfo {
     int64_t base;     // offset of the instance's first request
     int64_t sum_a;    // sum of arrival steps (TEL = sum of completions - sum_a)
     int64_t cap;      // step cap
-    int64_t work;     // cost estimate used to order instances (longest first)
     int32_t n;        // number of requests
     int32_t status;   // 0 or a sim_status from validation
     int32_t lmax;     // largest u_i or o_i of the instance (bounds every projected length)

@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
     const int inst = blockIdx.x;
     const int64_t base = S.off[inst];
     const int n = int(S.off[inst + 1] - base);
-    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, work = 0, lmax = 0;
+    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0;
     const bool in_smem = n <= kStageSmemN;
     QEnt *R = in_smem ? reinterpret_cast<QEnt *>(stage_smem) : S.rec + base;
     int32_t *RA = in_smem ? reinterpret_cast<int32_t *>(stage_smem + size_t(kStageSmemN) * sizeof(QEnt))
@@ -129,13 +129,11 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
         sum_a += a;
         sum_o += o;
         lmax = max(lmax, int64_t(max(u, o)));
-        work += int64_t(s) * o + int64_t(o) * o / 2;
     }
     bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
     bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
     sum_a = block_reduce<int64_t>(sum_a, sh64, false);
     sum_o = block_reduce<int64_t>(sum_o, sh64, false);
-    work = block_reduce<int64_t>(work, sh64, false);
     lmax = block_reduce<int64_t>(lmax, sh64, true);
     int status = ST_OK;
     if (bad_inval) status = ST_INVAL;
@@ -147,7 +145,6 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
         in.status = status;
         in.sum_a = sum_a;
         in.cap = S.step_cap > 0 ? S.step_cap : 64 * (int64_t(n) + sum_o);
-        in.work = work;
         in.lmax = int32_t(lmax);
         in.pad = 0;
         S.info[inst] = in;
