@@ -220,3 +220,20 @@ def test_debug_checks_hold_and_change_nothing(pol):
         assert np.all(b["status"] == 0)
         for f in FIELDS:
             assert np.array_equal(a[f], b[f]), (pol, f)
+
+
+def test_largest_memory_limit():
+    """M = 2^26 (the largest the ABI accepts) with requests of up to ~2^25 tokens: the 32-bit
+    bound fails, so the 64-bit kernel runs every instance; results equal the oracle (which steps
+    every one of the ~10^8 batches)."""
+    from paper_2508_14544_gb300 import workloads as W
+    M = 1 << 26
+    parts = [dict(a=[0, 0, 5, 9], s=[1000, 7, 1, 1 << 20], l=[1, 5, 1 << 24, 3],
+                  u=[1 << 25, 9, 1 << 25, (1 << 25) - (1 << 20)], o=[1 << 24, 9, (1 << 24) + 3, 1 << 22]),
+             dict(a=[0], s=[(1 << 26) - 2], l=[1], u=[2], o=[2])]
+    w = W.concat_instances("maxm", M, parts)
+    for pol in (0, 1, 2, 4):
+        got, _ = gpu_run(pol, w)
+        ref = oracle_run(pol, w)
+        for f in FIELDS:
+            assert np.array_equal(got[f], ref[f]), (pol, f)
