@@ -54,7 +54,8 @@ typedef enum {
     SIM_OK = 0,
     SIM_E_INVAL = -1,      /* bad argument, or an instance with l > o, o > u, l < 1, s < 1, a < 0 */
     SIM_E_INFEASIBLE = -2, /* an instance has a request with s + o > M (or s + u > M under A_max, A_ell) */
-    SIM_E_STEPCAP = -3,    /* an instance processed step_cap batches without finishing */
+    SIM_E_STEPCAP = -3,    /* an instance processed step_cap batches without finishing, or its step
+                              counter reached 2^31 - 2^27 (2^30 under A_ell) */
     SIM_E_CUDA = -4,       /* a CUDA runtime call failed; see sim_last_error */
     SIM_E_STATE = -5,      /* call out of order (e.g. sim_run before sim_load), or an internal check failed */
     SIM_E_NOMEM = -6       /* host or device allocation failed */

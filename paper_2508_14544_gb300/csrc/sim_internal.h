@@ -4,12 +4,17 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <climits>
+
 namespace simgb {
 
 // Internal per-instance status: the active set outgrew the per-instance capacity of the launch;
 // the host re-runs such instances with a larger, global-memory workspace.
 constexpr int32_t kStatusCapacity = -100;
 constexpr int64_t kMaxM = int64_t(1) << 26;
+// Steps are int32: an instance stops with SIM_E_STEPCAP before a step passes kMaxStep, which leaves
+// room for a projected length (<= M <= 2^26) on top of any step.
+constexpr int32_t kMaxStep = INT32_MAX - (int32_t(1) << 27);
 // A_ell queue keys are 2 a (arrival) and 2 t + 1 (promotion at step t): steps stay below 2^30.
 constexpr int32_t kAellMaxStep = (int32_t(1) << 30) - 1;
 

@@ -958,7 +958,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             status = ST_STATE;  // a consistency check of SIM_OPT_DEBUG_CHECKS failed
             break;
         }
-        if (steps >= cap) {
+        if (steps >= cap || t > kMaxStep) {
             status = ST_STEPCAP;
             break;
         }
@@ -1168,6 +1168,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             if (POL == P_AMIN && A > 0) tau = min(tau, int64_t(tb) + floor_div32(M - SB0, A) + 1);
             if (POL == P_AELL && A > 0) tau = min(tau, int64_t(w.E[0]) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
+            tau = min(tau, int64_t(kMaxStep) + 1);
             if (tau > int64_t(t) + 1 && hvalid && A > 0)
                 tau = min(tau, first_fit_step<N>(w, A, tb, SB0, M, t, h.s, h.key, tau));
             const int64_t c = max(tau - int64_t(t), int64_t(1));

@@ -237,3 +237,24 @@ def test_largest_memory_limit():
         ref = oracle_run(pol, w)
         for f in FIELDS:
             assert np.array_equal(got[f], ref[f]), (pol, f)
+
+
+def test_step_counter_limit_is_a_step_cap():
+    """Steps are 32-bit: an instance whose steps would pass 2^31 - 2^27 (2^30 under A_ell) stops
+    with SIM_E_STEPCAP instead of wrapping; instances far from the limit are unaffected."""
+    from paper_2508_14544_gb300 import workloads as W
+    near = (1 << 31) - (1 << 27) - 50
+    parts = [dict(a=[near, near], s=[1, 1], l=[10, 10], u=[100, 100], o=[100, 90]),
+             dict(a=[0, 3], s=[1, 2], l=[1, 1], u=[5, 5], o=[4, 5])]
+    w = W.concat_instances("late", 1000, parts)
+    ref = oracle_run(0, w)
+    for pol in (0, 1, 2):
+        got, _ = gpu_run(pol, w)
+        assert got["status"].tolist() == [-3, 0], pol
+        r = oracle_run(pol, w)
+        for f in FIELDS:
+            assert got[f][1] == r[f][1]
+    late = W.concat_instances("late_ell", 1000, [dict(a=[(1 << 30) - 5], s=[1], l=[10], u=[100], o=[100])])
+    got, _ = gpu_run(4, late)
+    assert got["status"].tolist() == [-3]
+    del ref
