@@ -1,6 +1,7 @@
 """Build libsim.so (the CUDA simulator behind include/sim.h) in-tree with nvcc for sm_103a."""
 from __future__ import annotations
 
+import fcntl
 import os
 import shutil
 import subprocess
@@ -33,10 +34,23 @@ def _stale() -> bool:
 
 
 def build(force: bool = False, verbose: bool = False, extra: list[str] | None = None) -> Path:
-    """Compile the two translation units in parallel and link the shared library."""
+    """Compile the translation units in parallel and link the shared library.  Safe to call from
+    several processes at once (e.g. every rank of a multi-GPU launch): one builds under a file
+    lock, the others wait and then find the library up to date."""
     if not force and not _stale():
         return LIB
     BUILD.mkdir(parents=True, exist_ok=True)
+    with open(BUILD / ".lock", "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            if not force and not _stale():
+                return LIB
+            return _build_locked(verbose, extra)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose: bool, extra: list[str] | None) -> Path:
     cc = nvcc()
     common = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", f"-I{INCLUDE}", f"-I{CSRC}",
                      "--expt-relaxed-constexpr"] + (extra or [])
