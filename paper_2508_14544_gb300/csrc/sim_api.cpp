@@ -231,6 +231,7 @@ static int load_impl(sim_ctx *c, const int64_t *offsets, const int32_t *a, const
     sp.policy = c->policy;
     sp.M = c->M;
     sp.n_inst = c->n_inst;
+    sp.n_max = int32_t(n_max);
     sp.step_cap = c->step_cap;
     sp.off = c->d_off;
     sp.a = c->d_raw;

@@ -47,6 +47,7 @@ struct StageParams {
     int policy;
     int64_t M;
     int32_t n_inst;
+    int32_t n_max;             // largest instance (sizes the staging kernel's shared memory; 0: unknown)
     int64_t step_cap;          // 0: default 64 * (n + sum o)
     const int64_t *off;        // n_inst + 1
     const int32_t *a, *s, *l, *u, *o;  // raw copies, n_total each

@@ -128,6 +128,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     sp.policy = policy;
     sp.M = M;
     sp.n_inst = n_instances;
+    sp.n_max = int32_t(n_max);
     sp.step_cap = 0;
     sp.off = d_off;
     sp.a = arrival_t;

@@ -44,32 +44,16 @@ __device__ T block_reduce(T v, T *sh, bool is_max) {
     return acc;
 }
 
-// Bitonic sort of n records by (a, key, idx) in place, padded virtually to a power of two
-// (positions >= n take no part).  R/RA are shared or global memory.
+// Bitonic sort of n records by (a, key, idx) in place in global memory, padded virtually to a
+// power of two (positions >= n take no part): instances too large for shared memory.
 __device__ void bitonic_sort(QEnt *R, int32_t *RA, int n) {
     int N = 1;
     while (N < n) N <<= 1;
     for (int k = 2; k <= N; k <<= 1) {
-        for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
-            const int half = k >> 1;
-            const int i = (p / half) * k + (p % half);
-            const int j = i ^ (k - 1);
-            if (j < n) {
-                const QEnt x = R[i], y = R[j];
-                const int ax = RA[i], ay = RA[j];
-                if (stage_less(ay, y, ax, x)) {
-                    R[i] = y;
-                    R[j] = x;
-                    RA[i] = ay;
-                    RA[j] = ax;
-                }
-            }
-        }
-        __syncthreads();
-        for (int d = k >> 2; d >= 1; d >>= 1) {
+        for (int d = k >> 1; d >= 1; d >>= 1) {
             for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
                 const int i = (p / d) * 2 * d + (p % d);
-                const int j = i + d;
+                const int j = (d == (k >> 1)) ? (i | (k - 1)) - (i & (k - 1)) : i + d;  // first pass: mirror
                 if (j < n) {
                     const QEnt x = R[i], y = R[j];
                     const int ax = RA[i], ay = RA[j];
@@ -86,20 +70,49 @@ __device__ void bitonic_sort(QEnt *R, int32_t *RA, int n) {
     }
 }
 
+// The same order for an instance held in shared memory as 12-byte pairs: the key (a << 32 | policy
+// key; both are >= 0 in a valid instance, so the unsigned order is the (a, key) order) and the
+// request index; the prompt and true lengths stay in place, indexed by request.
+__device__ __forceinline__ void bitonic_sort_pairs(uint64_t *sk, int32_t *si, int n) {
+    int N = 1;
+    while (N < n) N <<= 1;
+    for (int k = 2; k <= N; k <<= 1) {
+        for (int d = k >> 1; d >= 1; d >>= 1) {
+            for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
+                const int i = (p / d) * 2 * d + (p % d);
+                const int j = (d == (k >> 1)) ? (i | (k - 1)) - (i & (k - 1)) : i + d;
+                if (j < n) {
+                    const uint64_t ki = sk[i], kj = sk[j];
+                    const int ii = si[i], ij = si[j];
+                    if (kj < ki || (kj == ki && ij < ii)) {
+                        sk[i] = kj;
+                        sk[j] = ki;
+                        si[i] = ij;
+                        si[j] = ii;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
 // Instances of up to this many requests are sorted in shared memory (20 bytes per request).
 constexpr int kStageSmemN = 2048;
+constexpr int kStageSmemBytesPerReq = 20;
 
-__global__ void __launch_bounds__(256) k_stage(StageParams S) {
+__global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
     __shared__ int64_t sh64[32];
     extern __shared__ __align__(16) unsigned char stage_smem[];
     const int inst = blockIdx.x;
     const int64_t base = S.off[inst];
     const int n = int(S.off[inst + 1] - base);
     int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0;
-    const bool in_smem = n <= kStageSmemN;
-    QEnt *R = in_smem ? reinterpret_cast<QEnt *>(stage_smem) : S.rec + base;
-    int32_t *RA = in_smem ? reinterpret_cast<int32_t *>(stage_smem + size_t(kStageSmemN) * sizeof(QEnt))
-                          : S.rec_a + base;
+    const bool in_smem = n <= np;
+    uint64_t *sk = reinterpret_cast<uint64_t *>(stage_smem);
+    int32_t *si = reinterpret_cast<int32_t *>(stage_smem + size_t(np) * 8);
+    int32_t *ss = si + np;
+    int32_t *so = ss + np;
     for (int j = threadIdx.x; j < n; j += blockDim.x) {
         const int64_t g = base + j;
         const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
@@ -119,13 +132,20 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
             if (a > kAellMaxStep) bad_inval = 1;
             S.lu[g] = make_int2(l, u);  // indexed by request: j == idx below
         }
-        QEnt e;
-        e.key = key;
-        e.idx = j;
-        e.s = s;
-        e.o = o;
-        R[j] = e;
-        RA[j] = a;
+        if (in_smem) {
+            sk[j] = (uint64_t(uint32_t(a)) << 32) | uint32_t(key);
+            si[j] = j;
+            ss[j] = s;
+            so[j] = o;
+        } else {
+            QEnt e;
+            e.key = key;
+            e.idx = j;
+            e.s = s;
+            e.o = o;
+            S.rec[g] = e;
+            S.rec_a[g] = a;
+        }
         sum_a += a;
         sum_o += o;
         lmax = max(lmax, int64_t(max(u, o)));
@@ -150,13 +170,22 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S) {
         S.info[inst] = in;
     }
     __syncthreads();
-    if (status == ST_OK && n > 1) bitonic_sort(R, RA, n);
-    if (in_smem) {
-        // write the (sorted, or for a rejected instance unsorted) records out
-        for (int j = threadIdx.x; j < n; j += blockDim.x) {
-            S.rec[base + j] = R[j];
-            S.rec_a[base + j] = RA[j];
-        }
+    if (!in_smem) {
+        if (status == ST_OK && n > 1) bitonic_sort(S.rec + base, S.rec_a + base, n);
+        return;
+    }
+    if (status == ST_OK && n > 1) bitonic_sort_pairs(sk, si, n);
+    // write the (sorted, or for a rejected instance unsorted) records out
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+        const uint64_t k = sk[j];
+        const int idx = si[j];
+        QEnt e;
+        e.key = int(uint32_t(k));
+        e.idx = idx;
+        e.s = ss[idx];
+        e.o = so[idx];
+        S.rec[base + j] = e;
+        S.rec_a[base + j] = int(uint32_t(k >> 32));
     }
 }
 
@@ -174,8 +203,12 @@ __global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out,
 
 cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
     if (p.n_inst <= 0) return cudaSuccess;
-    const size_t smem = size_t(kStageSmemN) * (sizeof(QEnt) + sizeof(int32_t));  // 40 KB
-    k_stage<<<p.n_inst, 256, smem, st>>>(p);
+    // shared memory for the largest instance up to kStageSmemN, rounded up to a power of two
+    int np = 1;
+    const int want = (p.n_max > 0 && p.n_max < kStageSmemN) ? p.n_max : kStageSmemN;
+    while (np < want) np <<= 1;
+    const size_t smem = size_t(np) * kStageSmemBytesPerReq;
+    k_stage<<<p.n_inst, 256, smem, st>>>(p, np);
     return cudaGetLastError();
 }
 
