@@ -1,6 +1,7 @@
 """Command-line runner: simulate a named synthetic workload under one policy through the C ABI.
 
   python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024] [--repeat 1]
+                                       [--warps-per-block W] [--warps-per-sm S]
 
 Prints one JSON line per run with the wall time of sim_run, totals of the result fields, the
 throughput and a sha256 of the per-instance result records (equal across runs and launch shapes).
@@ -25,6 +26,7 @@ def main(argv=None) -> None:
     ap.add_argument("--instances", default=None, help="a:b range of instance ids (default: all)")
     ap.add_argument("--repeat", type=int, default=1)
     ap.add_argument("--warps-per-block", type=int, default=0)
+    ap.add_argument("--warps-per-sm", type=int, default=0, help="residency limit (4: one warp per scheduler)")
     args = ap.parse_args(argv)
     ids = None
     if args.instances:
@@ -37,6 +39,8 @@ def main(argv=None) -> None:
     opts = {}
     if args.warps_per_block:
         opts["warps_per_block"] = args.warps_per_block
+    if args.warps_per_sm:
+        opts["warps_per_sm"] = args.warps_per_sm
     with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
         for _ in range(args.repeat):
             sim.load(w.offsets, *dev, rank=rank)
@@ -51,6 +55,8 @@ def main(argv=None) -> None:
                               "request_steps_per_s": rs / dt, "steps_per_s": st / dt,
                               "total_latency": int(res["total_latency"].sum()),
                               "evictions": int(res["evictions"].sum()),
+                              "most_evictions": [int(ids[0] if ids else 0) + int(np.argmax(res["evictions"])),
+                                                 int(res["evictions"].max())],
                               "worst_status": int(res["status"].min()), "results_sha256": digest}), flush=True)
 
 
