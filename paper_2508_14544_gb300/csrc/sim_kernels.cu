@@ -117,6 +117,21 @@ __device__ __forceinline__ int excl_scan_add(int v, int &total) {
     return x - v;
 }
 
+// Exclusive count over lanes of the entries marked in lv (four per lane, entry 4 lane + j), by one
+// ballot per slot; total = all marked entries.
+__device__ __forceinline__ int excl_count4(const bool (&lv)[4], int &total) {
+    const unsigned lt = (1u << lane_id()) - 1u;
+    int off = 0, tot = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const unsigned b = __ballot_sync(FULL, lv[j]);
+        off += __popc(b & lt);
+        tot += __popc(b);
+    }
+    total = tot;
+    return off;
+}
+
 // Sum over lanes above this one; total = sum over all lanes.
 __device__ __forceinline__ int excl_suffix_add(int v, int &total) {
     const int lane = lane_id();
@@ -162,6 +177,39 @@ __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
         if (k < 32) break;
     }
     return cnt;
+}
+
+// #{i < len : E[i] <= y} and #{i < len : E[i] < y} for E ascending, searched in step (a
+// coarse round over 32 splitters, then one fine round each).
+__device__ __forceinline__ void prefix_le_lt(const int32_t *E, int len, int64_t y, int &hi, int &lb) {
+    hi = lb = 0;
+    if (len <= 0) return;
+    const int lane = lane_id();
+    const int c = (len + 31) >> 5;
+    const int e = E[min((lane + 1) * c - 1, len - 1)];
+    int h = min(__popc(__ballot_sync(FULL, e <= y)) * c, len);
+    int l = min(__popc(__ballot_sync(FULL, e < y)) * c, len);
+    const int eh = min(h + c, len), el = min(l + c, len);
+    bool dh = h >= len, dl = l >= len;
+    int oh = h, ol = l;
+    while (!(dh && dl)) {
+        const int ih = oh + lane, il = ol + lane;
+        const bool ph = !dh && ih < eh && E[ih] <= y;
+        const bool pl = !dl && il < el && E[il] < y;
+        const int kh = __popc(__ballot_sync(FULL, ph)), kl = __popc(__ballot_sync(FULL, pl));
+        if (!dh) {
+            h += kh;
+            oh += 32;
+            dh = kh < 32 || oh >= eh;
+        }
+        if (!dl) {
+            l += kl;
+            ol += 32;
+            dl = kl < 32 || ol >= el;
+        }
+    }
+    hi = h;
+    lb = l;
 }
 
 // The same, computed by one lane alone (binary search).
@@ -484,6 +532,57 @@ __device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int
     __syncwarp();
 }
 
+// One-chunk sets (0 < A <= kChunk) after an insertion: derive() in one pass, the suffix sums kept
+// in registers for the prefix maxima.
+template <bool N>
+__device__ __forceinline__ void derive_one(const Ws &w, int A, int tb, int &SB0, int &nextF) {
+    const int lane = lane_id();
+    {
+        const int base = 4 * lane;
+        const int4 b4 = ld4(w.B, base), e4 = ld4(w.E, base), f4 = ld4(w.F, base);
+        const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, ee[4] = {e4.x, e4.y, e4.z, e4.w};
+        const int ff[4] = {f4.x, f4.y, f4.z, f4.w};
+        int s[4];
+        int acc = 0;
+#pragma unroll
+        for (int j = 3; j >= 0; --j) {
+            acc += (base + j < A) ? bb[j] + tb : 0;
+            s[j] = acc;
+        }
+        int tot;
+        const int after = excl_suffix_add(acc, tot);
+        int m[4];
+        int mx = INT_MIN, fmin = INT_MAX;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            int h = INT_MIN;
+            if (base + j < A) {
+                const wint<N> e = wint<N>(ee[j]) - tb;
+                h = satw<N>(wint<N>(s[j] + after) + wint<N>(A - base - j) * e + e);
+                fmin = min(fmin, ff[j]);
+            }
+            mx = max(mx, h);
+            m[j] = mx;
+        }
+        const int before = excl_scan_max(mx);
+        nextF = __reduce_min_sync(FULL, fmin);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (base + j < A) {
+                w.SB[base + j] = s[j] + after;
+                w.PM[base + j + 1] = max(before, m[j]);
+            }
+        }
+        if (lane == 0) {
+            w.SB[A] = 0;
+            w.PM[0] = INT_MIN;
+        }
+        SB0 = tot;
+        __syncwarp();
+        return;
+    }
+}
+
 // Remove the entries marked dead (F < 0), keeping the order; entries only move left.
 __device__ __forceinline__ void compact(const Ws &w, int &A) {
     const int lane = lane_id();
@@ -503,7 +602,7 @@ __device__ __forceinline__ void compact(const Ws &w, int &A) {
             lc += lv[j] ? 1 : 0;
         }
         int L;
-        const int off = excl_scan_add(lc, L);
+        const int off = excl_count4(lv, L);
         __syncwarp();
         int qd = wpos + off;
 #pragma unroll
@@ -540,7 +639,7 @@ __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int 
         lc += lv[j] ? 1 : 0;
     }
     int L;
-    const int off = excl_scan_add(lc, L);
+    const int off = excl_count4(lv, L);
     int sfx[4];
     int acc = 0;
 #pragma unroll
@@ -1078,8 +1177,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
             if (fits && A > 0) {
                 const int64_t y = int64_t(t) + h.key - 1;
                 if (pdirty || y != y_prev + 1) {
-                    hi = warp_prefix_count(A, [&](int i) { return w.E[i] <= y; });
-                    lb = warp_prefix_count(hi, [&](int i) { return w.E[i] < y; });
+                    prefix_le_lt(w.E, A, y, hi, lb);
                 } else {
                     lb = hi;
                     while (hi < A && w.E[hi] <= y) ++hi;
@@ -1119,7 +1217,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                 break;
             }
             tb = t;
-            derive<N>(w, A, tb, SB0, nextF);
+            if (A <= kChunk) derive_one<N>(w, A, tb, SB0, nextF);
+            else derive<N>(w, A, tb, SB0, nextF);
             pdirty = true;
             if (Kadm < W) {
                 // window entry Kadm is the new head, and it does not fit at step t
