@@ -992,9 +992,13 @@ __device__ bool state_ok(const Ws &w, const Queue &q, int A, int tb, int SB0, in
 // One instance, simulated by one warp.  All lanes hold identical copies of the scalar state.
 // ---------------------------------------------------------------------------------------------
 template <int POL, bool N>
-__device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, int inst) {
+__device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, int inst) {
     const int lane = lane_id();
     const InstInfo info = P.info[inst];
+    // delta capacity for this instance: shifts in the delta cost O(capacity) per insertion, merges
+    // into the main array O(n) per capacity insertions; a small delta suits a short queue
+    Ws w = w0;
+    w.dcap = info.n <= 1024 ? min(w0.dcap, 64) : (info.n <= 4096 ? min(w0.dcap, 128) : w0.dcap);
     DevResult r;
     r.total_latency = r.makespan = r.peak_memory = r.evictions = r.steps = r.request_steps = 0;
     r.status = info.status;
@@ -1110,12 +1114,11 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w, in
                     }
                     const unsigned mk = __reduce_min_sync(FULL, bk);
                     const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
-                    const unsigned ball = __ballot_sync(FULL, bp >= 0 && bk == mk && bi == mi);
-                    if (ball == 0) {
+                    const int pos = int(__reduce_min_sync(FULL, (bp >= 0 && bk == mk && bi == mi) ? unsigned(bp) : UINT_MAX));
+                    if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
                         break;
                     }
-                    const int pos = __shfl_sync(FULL, bp, __ffs(ball) - 1);
                     const int b = w.B[pos], p = w.P[pos], f = w.F[pos], k = w.K[pos], id = w.I[pos];
                     QEnt e;
                     e.key = max(k, t - p);  // refined lower bound: max(estimate, tokens generated)
