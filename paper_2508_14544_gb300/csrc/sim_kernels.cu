@@ -163,6 +163,11 @@ template <class Pred>
 __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
     if (len <= 0) return 0;
     const int lane = lane_id();
+    if (len <= 64) {  // two entries per lane: one round
+        const bool p0 = lane < len && pred(lane);
+        const bool p1 = lane + 32 < len && pred(lane + 32);
+        return __popc(__ballot_sync(FULL, p0)) + __popc(__ballot_sync(FULL, p1));
+    }
     const int c = (len + 31) >> 5;
     const int pos = min((lane + 1) * c - 1, len - 1);
     const int full = __popc(__ballot_sync(FULL, pred(pos)));
