@@ -692,11 +692,12 @@ __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int 
 // cnt_m = #{old E <= E_m}, new entry m goes to m + cnt_m and old entry p moves right by
 // #{m : cnt_m <= p}.  Entries only move right, so chunks are processed from the back.
 // Returns false if the capacity is exceeded.
-__device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t, const QEnt &mine) {
+__device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t, const QEnt &mine, int le) {
     const int lane = lane_id();
     if (A + K > w.ca) return false;
     const int ne = t + mine.key - 1;
-    const int cnt = (lane < K) ? lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; }) : INT_MAX;
+    // le >= 0: #{old E <= E_m} already found by the admission test
+    const int cnt = (lane < K) ? (le >= 0 ? le : lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; })) : INT_MAX;
     const int last = ((A - 1) / kChunk) * kChunk;
     for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
         const int base = cb + 4 * lane;
@@ -796,7 +797,8 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
 // k at which any point exceeds M ends the prefix.  Falls back to the binary-search form otherwise.
 template <bool N>
 __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int W,
-                                                 const QEnt &mine) {
+                                                 const QEnt &mine, int &le) {
+    le = -1;
     if (A > kChunk) return admissible_prefix_search<N>(w, A, tb, SB0, M, t, W, mine);
     const int lane = lane_id();
     const int Mi = int(M);
@@ -817,8 +819,22 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     int vc = INT_MIN;
     int av = 0;
     if (lane < W) {
-        const int64_t y = int64_t(t) + dm;
-        const int lb = lane_prefix_count(A, [&](int i) { return int64_t(w.E[i]) < y; });
+        // #{E < y} for V(y), and #{E <= y}, where the entry goes if it is admitted (insert_window),
+        // by two binary searches in step
+        const int y = t + dm;
+        int lo1 = 0, hi1 = A, lo2 = 0, hi2 = A;
+        while (lo1 < hi1 || lo2 < hi2) {
+            const int m1 = (lo1 + hi1) >> 1, m2 = (lo2 + hi2) >> 1;
+            const int e1 = w.E[min(m1, A - 1)], e2 = w.E[min(m2, A - 1)];
+            if (lo1 < hi1) {
+                if (e1 < y) lo1 = m1 + 1; else hi1 = m1;
+            }
+            if (lo2 < hi2) {
+                if (e2 <= y) lo2 = m2 + 1; else hi2 = m2;
+            }
+        }
+        const int lb = lo1;
+        le = lo2;
         av = satw<N>(wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb));
     }
     wint<N> need = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
@@ -1208,9 +1224,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (POL == P_AR || POL == P_AELL) {
                 if (lane < W) mine = proj<POL>(P, info.base, mine);
             }
+            int le = -1;
             const int Kadm = (POL == P_AR || POL == P_AELL)
                                  ? admissible_prefix_general<N>(w, A, tb, SB0, M, t, W, mine)
-                                 : admissible_prefix<N>(w, A, tb, SB0, M, t, W, mine);
+                                 : admissible_prefix<N>(w, A, tb, SB0, M, t, W, mine, le);
             if (Kadm <= 0) {
                 status = ST_STATE;  // the head test and the window disagree: internal error
                 break;
@@ -1220,7 +1237,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             q.dn -= Kadm - cm;
             // entries >= Kadm stay in their lanes, so the new head below is unaffected
             if ((POL == P_AR || POL == P_AELL) && Kadm > 1) sort_admitted(w, Kadm, mine);
-            if (!insert_window(w, A, Kadm, t, mine)) {
+            if (!insert_window(w, A, Kadm, t, mine, le)) {
                 status = kStatusCapacity;
                 break;
             }
