@@ -1034,6 +1034,12 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         return;
     }
     const int n = info.n;
+    // A_min cancellation order (estimate, index) as one 32-bit key when both fit: index bits kib
+    int kib = -1;
+    if (POL == P_AMIN) {
+        const int ib = 32 - __clz(max(n - 1, 1));
+        if (ib < 31 && (int64_t(info.lmax) + 1) <= (int64_t(1) << (32 - ib)) - 1) kib = ib;
+    }
     const QEnt *rec = P.rec + info.base;
     const int32_t *ra = P.rec_a + info.base;
     const int64_t M = P.M;
@@ -1114,28 +1120,53 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
             if (need > wint<N>(M)) {
                 while (need > wint<N>(M)) {
-                    unsigned bk = UINT_MAX, bi = UINT_MAX;
-                    int bp = -1;
-                    for (int cb = 0; cb < A; cb += kChunk) {
-                        const int base = cb + 4 * lane;
-                        const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
-                        const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-                        const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
+                    int pos;
+                    if (kib >= 0) {
+                        // (estimate, index) packed into one 32-bit key: one reduction for the minimum
+                        unsigned best = UINT_MAX;
+                        int bp = -1;
+                        for (int cb = 0; cb < A; cb += kChunk) {
+                            const int base = cb + 4 * lane;
+                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                            const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            if (base + j < A && ff[j] >= 0) {
-                                const unsigned k = unsigned(kk[j]), i = unsigned(ii[j]);
-                                if (k < bk || (k == bk && i < bi)) {
-                                    bk = k;
-                                    bi = i;
+                            for (int j = 0; j < 4; ++j) {
+                                const unsigned key = (base + j < A && ff[j] >= 0)
+                                                         ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
+                                                         : UINT_MAX;
+                                if (key < best) {
+                                    best = key;
                                     bp = base + j;
                                 }
                             }
                         }
+                        const unsigned mk = __reduce_min_sync(FULL, best);
+                        pos = int(__reduce_min_sync(FULL, (bp >= 0 && best == mk) ? unsigned(bp) : UINT_MAX));
+                    } else {
+                        unsigned bk = UINT_MAX, bi = UINT_MAX;
+                        int bp = -1;
+                        for (int cb = 0; cb < A; cb += kChunk) {
+                            const int base = cb + 4 * lane;
+                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                            const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                if (base + j < A && ff[j] >= 0) {
+                                    const unsigned k = unsigned(kk[j]), i = unsigned(ii[j]);
+                                    if (k < bk || (k == bk && i < bi)) {
+                                        bk = k;
+                                        bi = i;
+                                        bp = base + j;
+                                    }
+                                }
+                            }
+                        }
+                        const unsigned mk = __reduce_min_sync(FULL, bk);
+                        const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
+                        pos = int(__reduce_min_sync(FULL, (bp >= 0 && bk == mk && bi == mi) ? unsigned(bp) : UINT_MAX));
                     }
-                    const unsigned mk = __reduce_min_sync(FULL, bk);
-                    const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
-                    const int pos = int(__reduce_min_sync(FULL, (bp >= 0 && bk == mk && bi == mi) ? unsigned(bp) : UINT_MAX));
                     if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
                         break;
