@@ -1125,6 +1125,23 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                         // (estimate, index) packed into one 32-bit key: one reduction for the minimum
                         unsigned best = UINT_MAX;
                         int bp = -1;
+                        if (A <= kChunk) {
+                            // one chunk: a min tree over this lane's four keys, then the position
+                            const int base = 4 * lane;
+                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                            const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
+                            unsigned key[4];
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                key[j] = (base + j < A && ff[j] >= 0) ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
+                                                                     : UINT_MAX;
+                            best = min(min(key[0], key[1]), min(key[2], key[3]));
+                            const unsigned mk = __reduce_min_sync(FULL, best);
+                            const int j = key[0] == mk ? 0 : (key[1] == mk ? 1 : (key[2] == mk ? 2 : 3));
+                            bp = (best == mk && mk != UINT_MAX) ? base + j : -1;
+                            pos = int(__reduce_min_sync(FULL, bp >= 0 ? unsigned(bp) : UINT_MAX));
+                        } else {
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
                             const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
@@ -1143,6 +1160,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                         }
                         const unsigned mk = __reduce_min_sync(FULL, best);
                         pos = int(__reduce_min_sync(FULL, (bp >= 0 && best == mk) ? unsigned(bp) : UINT_MAX));
+                        }
                     } else {
                         unsigned bk = UINT_MAX, bi = UINT_MAX;
                         int bp = -1;
