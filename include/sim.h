@@ -89,12 +89,22 @@ enum {
     SIM_OPT_WARPS_PER_SM = 5,       /* 0..64: at most this many simulation warps resident per SM
                                        (0, the default: as many as shared memory allows).  Results
                                        do not depend on it. */
-    SIM_OPT_DEBUG_CHECKS = 6        /* 0/1: run every instance in the global-memory kernel and check
+    SIM_OPT_DEBUG_CHECKS = 6,       /* 0/1: run every instance in the global-memory kernel and check
                                        the simulation state's invariants between events (active set
                                        sorted by projected end, suffix sums and prefix maxima of the
                                        set, queue order; no job past its projected end under A_max,
                                        H-SF and A_r).  A violation gives that instance SIM_E_STATE.
                                        Slower; results are otherwise identical. */
+    SIM_OPT_TUNE_RESIDENCY = 7      /* 0/1: on the first sim_run of a load shape (n_instances, total
+                                       and largest instance size), time the simulation launch with
+                                       one warp per scheduler (4 per SM) and with the default
+                                       residency, and use the faster for every later sim_run of
+                                       that shape, across sim_load calls (default 0).  A launch is
+                                       as long as its slowest instance: one warp per scheduler
+                                       wins when a few instances dominate (A_min with long
+                                       cancellation chains), two when instances are even.  The
+                                       tuning run simulates twice; results do not depend on it.
+                                       Overrides SIM_OPT_WARPS_PER_SM while set. */
 };
 
 /*

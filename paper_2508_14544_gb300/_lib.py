@@ -18,6 +18,7 @@ SIM_OK, SIM_E_INVAL, SIM_E_INFEASIBLE, SIM_E_STEPCAP, SIM_E_CUDA, SIM_E_STATE, S
 SIM_OPT_STEP_CAP, SIM_OPT_RECORD_COMPLETIONS, SIM_OPT_WARPS_PER_BLOCK, SIM_OPT_SMEM_ACTIVE_CAP = 1, 2, 3, 4
 SIM_OPT_WARPS_PER_SM = 5
 SIM_OPT_DEBUG_CHECKS = 6
+SIM_OPT_TUNE_RESIDENCY = 7
 
 STATUS_NAMES = {0: "SIM_OK", -1: "SIM_E_INVAL", -2: "SIM_E_INFEASIBLE", -3: "SIM_E_STEPCAP", -4: "SIM_E_CUDA",
                 -5: "SIM_E_STATE", -6: "SIM_E_NOMEM"}

@@ -30,6 +30,11 @@ struct sim_ctx {
     int wpb = 4;
     int warps_per_sm = 0;
     int debug_checks = 0;
+    int tune_residency = 0;
+    // residency chosen by SIM_OPT_TUNE_RESIDENCY for the load shape tuned_shape (n_inst, n_total,
+    // n_max): warps per SM, or 0 for the default; tuned_shape[0] < 0 when not tuned
+    int tuned_wps = 0;
+    int64_t tuned_shape[3] = {-1, -1, -1};
     int smem_ca = 512;
     int dcap = 256;
     // state
@@ -159,6 +164,10 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
         case SIM_OPT_DEBUG_CHECKS:
             c->debug_checks = value ? 1 : 0;
             return SIM_OK;
+        case SIM_OPT_TUNE_RESIDENCY:
+            c->tune_residency = value ? 1 : 0;
+            c->tuned_shape[0] = -1;
+            return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
             if (value < 128 || value > 4096 || value % 128)
                 return fail(c, SIM_E_INVAL, "SMEM_ACTIVE_CAP must be a multiple of 128 in [128, 4096]");
@@ -275,7 +284,8 @@ int sim_load(sim_ctx *c, int32_t n, const int32_t *a, const int32_t *s, const in
     return sim_load_csr(c, off.data(), a, s, l, u, o, device_ptrs);
 }
 
-static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int32_t n_work, bool smem) {
+static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int32_t n_work, bool smem,
+                      int warps_per_sm) {
     cudaError_t e;
     int dev = c->device;
     int n_sm = 0, smem_optin = 0;
@@ -302,7 +312,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     } else {
         per_sm = std::max(1, 16 / wpb);
     }
-    if (c->warps_per_sm > 0) per_sm = std::max(1, std::min(per_sm, c->warps_per_sm / wpb));
+    if (warps_per_sm > 0) per_sm = std::max(1, std::min(per_sm, warps_per_sm / wpb));
     int64_t blocks = int64_t(n_sm) * per_sm;
     blocks = std::min<int64_t>(blocks, (n_work + wpb - 1) / wpb);
     blocks = std::max<int64_t>(blocks, 1);
@@ -370,8 +380,39 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
             return cuda_fail(c, e, "cudaMemsetAsync");
     }
     // with SIM_OPT_DEBUG_CHECKS every instance runs in the checking global-memory kernel
-    rc = run_launch(c, st, nullptr, c->n_inst, !c->debug_checks);
-    if (rc) return rc;
+    int wps = c->warps_per_sm;
+    bool simulated = false;  // a tuning launch already wrote the results (they do not depend on residency)
+    if (c->tune_residency && !c->debug_checks) {
+        const int64_t shape[3] = {c->n_inst, c->n_total, c->n_max};
+        if (!std::equal(shape, shape + 3, c->tuned_shape)) {
+            // one warp per scheduler (4 schedulers per SM) against the default, timed on the stream
+            cudaEvent_t ev[3];
+            for (auto &x : ev)
+                if ((e = cudaEventCreate(&x)) != cudaSuccess) return cuda_fail(c, e, "cudaEventCreate");
+            const int cand[2] = {4, 0};
+            float ms[2] = {0.f, 0.f};
+            cudaEventRecord(ev[0], st);
+            for (int k = 0; k < 2 && rc == SIM_OK; ++k) {
+                rc = run_launch(c, st, nullptr, c->n_inst, true, cand[k]);
+                cudaEventRecord(ev[k + 1], st);
+            }
+            if (rc == SIM_OK && (e = cudaEventSynchronize(ev[2])) == cudaSuccess) {
+                cudaEventElapsedTime(&ms[0], ev[0], ev[1]);
+                cudaEventElapsedTime(&ms[1], ev[1], ev[2]);
+                c->tuned_wps = ms[0] < ms[1] ? cand[0] : cand[1];
+                std::copy(shape, shape + 3, c->tuned_shape);
+                simulated = true;
+            }
+            for (auto &x : ev) cudaEventDestroy(x);
+            if (rc) return rc;
+            if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: residency tuning");
+        }
+        wps = c->tuned_wps;
+    }
+    if (!simulated) {
+        rc = run_launch(c, st, nullptr, c->n_inst, !c->debug_checks, wps);
+        if (rc) return rc;
+    }
     c->h_res.resize(size_t(c->n_inst));
     e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost, st);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: copy of the results");
@@ -384,7 +425,7 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
     if (!redo.empty()) {
         e = cudaMemcpyAsync(c->d_work, redo.data(), redo.size() * sizeof(int32_t), cudaMemcpyHostToDevice, st);
         if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: work list");
-        rc = run_launch(c, st, c->d_work, int32_t(redo.size()), false);
+        rc = run_launch(c, st, c->d_work, int32_t(redo.size()), false, c->warps_per_sm);
         if (rc) return rc;
         e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost,
                             st);

@@ -22,7 +22,8 @@ class Simulator:
 
     OPTIONS = {"step_cap": L.SIM_OPT_STEP_CAP, "record_completions": L.SIM_OPT_RECORD_COMPLETIONS,
                "warps_per_block": L.SIM_OPT_WARPS_PER_BLOCK, "smem_active_cap": L.SIM_OPT_SMEM_ACTIVE_CAP,
-               "warps_per_sm": L.SIM_OPT_WARPS_PER_SM, "debug_checks": L.SIM_OPT_DEBUG_CHECKS}
+               "warps_per_sm": L.SIM_OPT_WARPS_PER_SM, "debug_checks": L.SIM_OPT_DEBUG_CHECKS,
+               "tune_residency": L.SIM_OPT_TUNE_RESIDENCY}
 
     def set_option(self, name: str, value: int) -> None:
         rc = L.sim_set_option(self.ctx, self.OPTIONS[name], int(value))

@@ -106,6 +106,41 @@ def test_launch_shapes_agree(wpb, wps):
             assert np.array_equal(a[f], b[f])
 
 
+def test_residency_tuning():
+    """SIM_OPT_TUNE_RESIDENCY: the first run of a load shape simulates with both residencies
+    (two simulation launches), later runs and reloads of the same shape launch once, a new shape
+    is tuned again, and no result changes."""
+    from paper_2508_14544_gb300 import POLICIES, Simulator
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(3, 1024, 17))
+    w2 = W.make_workload("c2", range(0, 1024, 29))
+    for pol in ("A_min", "A_max"):
+        ref, _ = gpu_run(POLICIES[pol], w)
+        ref2, _ = gpu_run(POLICIES[pol], w2)
+        with Simulator(POLICIES[pol], w.M, w.n_instances, tune_residency=1) as sim:
+            sim.load_workload(w)
+            k0 = sim.kernel_launches()
+            r1 = sim.run()
+            k1 = sim.kernel_launches()
+            r2 = sim.run()
+            k2 = sim.kernel_launches()
+            sim.load_workload(w)
+            k3 = sim.kernel_launches()
+            r3 = sim.run()
+            k4 = sim.kernel_launches()
+            assert (k1 - k0, k2 - k1, k4 - k3) == (2, 1, 1)
+            for r in (r1, r2, r3):
+                for f in FIELDS:
+                    assert np.array_equal(r[f], ref[f])
+        with Simulator(POLICIES[pol], w2.M, w2.n_instances, tune_residency=1) as sim:
+            sim.load_workload(w2)
+            k0 = sim.kernel_launches()
+            r = sim.run()
+            assert sim.kernel_launches() - k0 == 2
+            for f in FIELDS:
+                assert np.array_equal(r[f], ref2[f])
+
+
 def test_more_instances_than_warps():
     """One resident warp per SM (152 warps) for 342 instances: every warp simulates several
     instances in turn, reusing its workspace, and the results do not change."""
