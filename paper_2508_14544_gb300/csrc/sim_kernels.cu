@@ -18,7 +18,8 @@
 // Active set (per warp, shared memory; a global-memory workspace of the same layout serves
 // instances that outgrow it), structure of arrays sorted by the projected last step E:
 //   E = p + Lhat - 1   projected last step (Lhat = u, o or the A_min estimate)
-//   F = p + o - 1      true last step (completion at step F, C = F + 1); F < 0 marks a removed job
+//   F = p + o - 1      true last step (completion at step F, C = F + 1); F = -1 marks a cancelled
+//                      (A_min) or promoted (A_ell) job
 //   B = s - p + 1      the job's memory at step x is B + x
 //   P = p, I = request index, K = the estimate (A_min key)
 // Derived arrays, recomputed in one warp pass whenever the set changes, relative to a time base tb:
@@ -588,8 +589,9 @@ __device__ __forceinline__ void derive_one(const Ws &w, int A, int tb, int &SB0,
     }
 }
 
-// Remove the entries marked dead (F < 0), keeping the order; entries only move left.
-__device__ __forceinline__ void compact(const Ws &w, int &A) {
+// Remove the entries that ended before the new time base tb (completed at tb - 1, or marked with
+// F = -1), keeping the order; entries only move left.
+__device__ __forceinline__ void compact(const Ws &w, int &A, int tb) {
     const int lane = lane_id();
     int wpos = 0;
     for (int cb = 0; cb < A; cb += kChunk) {
@@ -603,7 +605,7 @@ __device__ __forceinline__ void compact(const Ws &w, int &A) {
         int lc = 0;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            lv[j] = (base + j < A) && ff[j] >= 0;
+            lv[j] = (base + j < A) && ff[j] >= tb;
             lc += lv[j] ? 1 : 0;
         }
         int L;
@@ -619,13 +621,13 @@ __device__ __forceinline__ void compact(const Ws &w, int &A) {
     A = wpos;
 }
 
-// Remove the entries marked dead (F < 0) and recompute the derived arrays, in one pass when the
+// Remove the entries with F < tb (see compact) and recompute the derived arrays, in one pass when the
 // set fits one chunk (positions, suffix sums and prefix maxima of the compacted order are known
 // from the live counts before anything is stored).
 template <bool N>
 __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int &SB0, int &nextF) {
     if (A > kChunk) {
-        compact(w, A);
+        compact(w, A, tb);
         derive<N>(w, A, tb, SB0, nextF);
         return;
     }
@@ -640,7 +642,7 @@ __device__ __forceinline__ void compact_derive(const Ws &w, int &A, int tb, int 
     int lc = 0;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-        lv[j] = (base + j < A) && ff[j] >= 0;
+        lv[j] = (base + j < A) && ff[j] >= tb;
         lc += lv[j] ? 1 : 0;
     }
     int L;
@@ -1072,7 +1074,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     int64_t y_prev = 0;
     int hi = 0, lb = 0;
 
-    bool pend_compact = false;
+    bool pend_compact = false, done_step = false;
     int tb_next = 0;
     for (;;) {
         if (pend_compact) {
@@ -1080,9 +1082,17 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             // removal share this one site: the loop body stays small, which matters when two
             // warps at different points of it share a scheduler's instruction cache.
             tb = tb_next;
+            const int A0 = A;
             compact_derive<N>(w, A, tb, SB0, nextF);
             pend_compact = false;
             pdirty = true;
+            if (done_step) {  // the jobs completed at step tb - 1 (C = tb) have left the set
+                const int c = A0 - A;
+                sumC += int64_t(c) * tb;
+                ndone += c;
+                done_step = false;
+                if (ndone >= n) break;
+            }
         }
         if (!N && P.debug && !state_ok<POL, N>(w, q, A, tb, SB0, nextF)) {
             status = ST_STATE;  // a consistency check of SIM_OPT_DEBUG_CHECKS failed
@@ -1316,22 +1326,17 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (mem > peak) peak = mem;
             rsteps += A;
             ++steps;
-            int c = 0;
-            for (int i = lane; i < A; i += 32) {
-                if (w.F[i] == t) {
-                    ++c;
-                    if (P.completion) P.completion[info.base + w.I[i]] = int64_t(t) + 1;
-                    w.F[i] = -1;
-                }
+            // the jobs with F = t complete (C = t + 1): the compaction at the top of the next
+            // iteration removes them (F < the new time base) and counts them
+            if (P.completion) {
+#pragma unroll 1
+                for (int i = lane; i < A; i += 32)
+                    if (w.F[i] == t) P.completion[info.base + w.I[i]] = int64_t(t) + 1;
             }
-            c = __reduce_add_sync(FULL, c);
-            __syncwarp();
-            sumC += int64_t(c) * (int64_t(t) + 1);
             makespan = int64_t(t) + 1;
-            ndone += c;
-            if (ndone >= n) break;
             tb_next = t + 1;
             pend_compact = true;
+            done_step = true;
             ++t;
         } else {
             // steps t .. tau-1 change nothing: no completion before nextF, no arrival before
