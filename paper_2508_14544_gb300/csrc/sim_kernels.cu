@@ -53,6 +53,9 @@ namespace {
 constexpr unsigned FULL = 0xffffffffu;
 enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2, P_AR = 3, P_AELL = 4 };
 enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
+// Loops whose trip count is known only at run time carry `#pragma unroll 1`: their unrolled copies
+// added 15-20 % to the code of the simulation loop, which two warps on one scheduler share through
+// its instruction cache.
 constexpr int kChunk = 128;  // active-set entries per warp pass (4 per lane)
 constexpr int kWin = 32;     // admission window (one candidate per lane)
 constexpr int kMc = 64;      // cached entries of the main queue (two per lane)
@@ -175,6 +178,7 @@ __device__ __forceinline__ int warp_prefix_count(int len, Pred pred) {
     int cnt = full * c;
     if (cnt >= len) return len;
     const int end = min(cnt + c, len);
+    #pragma unroll 1
     for (int off = cnt; off < end; off += 32) {
         const int i = off + lane;
         const unsigned b = __ballot_sync(FULL, i < end && pred(i));
@@ -198,6 +202,7 @@ __device__ __forceinline__ void prefix_le_lt(const int32_t *E, int len, int64_t 
     const int eh = min(h + c, len), el = min(l + c, len);
     bool dh = h >= len, dl = l >= len;
     int oh = h, ol = l;
+    #pragma unroll 1
     while (!(dh && dl)) {
         const int ih = oh + lane, il = ol + lane;
         const bool ph = !dh && ih < eh && E[ih] <= y;
@@ -222,6 +227,7 @@ __device__ __forceinline__ void prefix_le_lt(const int32_t *E, int len, int64_t 
 template <class Pred>
 __device__ __forceinline__ int lane_prefix_count(int len, Pred pred) {
     int lo = 0, hi = len;
+    #pragma unroll 1
     while (lo < hi) {
         const int mid = (lo + hi) >> 1;
         if (pred(mid)) lo = mid + 1; else hi = mid;
@@ -318,6 +324,7 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
     const int nx = q.me - q.mh;
     QEnt *out = (q.mbuf == 0) ? mb1 : mb0;
     const QEnt *X = q.mq + q.mh;
+    #pragma unroll 1
     for (int j = lane; j <= dn; j += 32) cnt[j] = 0;
     __syncwarp();
     const int c = (nx + 31) >> 5;
@@ -327,8 +334,10 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
         const QEnt x0 = X[s0];
         int r = lane_prefix_count(dn, [&](int m) { return qless(dq[dn - 1 - m], x0); });
         int run_r = r, run_len = 0;
+        #pragma unroll 1
         for (int i = s0; i < s1; ++i) {
             const QEnt x = X[i];
+            #pragma unroll 1
             while (r < dn && qless(dq[dn - 1 - r], x)) ++r;
             out[i + r] = x;
             if (r != run_r) {
@@ -343,6 +352,7 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
     __syncwarp();
     // delta element j (ascending) goes to j + #{main entries smaller} = j + sum_{r <= j} cnt[r]
     int carry = 0;
+    #pragma unroll 1
     for (int c0 = 0; c0 < dn; c0 += 32) {
         const int j = c0 + lane;
         int v = (j < dn) ? cnt[j] : 0;
@@ -378,6 +388,7 @@ __device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &
     if (q.dn == w.dcap) merge_delta(w, q);
     const int dn = q.dn;
     const int pos = warp_prefix_count(dn, [&](int i) { return qless(e, w.dq[i]); });  // #entries > e
+    #pragma unroll 1
     for (int hi = dn; hi > pos; hi -= 32) {
         const int lo = max(pos, hi - 32);
         const int i = lo + lane;
@@ -422,14 +433,17 @@ __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *ru
         return;
     }
     int done = 0;
+    #pragma unroll 1
     while (done < len) {
         const int rem = len - done;
         if (rem <= 8) {
+            #pragma unroll 1
             for (int j = 0; j < rem; ++j) delta_insert(w, q, run[done + j]);
             break;
         }
         if (q.dn > 0) merge_delta(w, q);
         const int k = min(rem, w.dcap);
+        #pragma unroll 1
         for (int j = lane; j < k; j += 32) w.dq[j] = run[done + k - 1 - j];  // descending
         __syncwarp();
         q.dn = k;
@@ -450,6 +464,7 @@ __device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, i
     const QEnt *A = w.mc + (q.mh - q.mcb);  // A[i], ascending
     const QEnt *Bd = w.dq + (dn - 1);       // B[j] = Bd[-j], ascending
     int lo = max(0, lane - nb), hi = min(lane, na);
+    #pragma unroll 1
     while (lo < hi) {
         const int mid = (lo + hi) >> 1;
         if (qless(A[mid], Bd[-(lane - 1 - mid)])) lo = mid + 1; else hi = mid;
@@ -483,6 +498,7 @@ __device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int
     const int lane = lane_id();
     int carry = 0;
     const int last = ((A - 1) / kChunk) * kChunk;
+    #pragma unroll 1
     for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
         const int base = cb + 4 * lane;
         const int4 b4 = ld4(w.B, base);
@@ -509,6 +525,7 @@ __device__ __forceinline__ void derive(const Ws &w, int A, int tb, int &SB0, int
     SB0 = carry;
     int run = INT_MIN;
     int fmin = INT_MAX;
+    #pragma unroll 1
     for (int cb = 0; cb < A; cb += kChunk) {
         const int base = cb + 4 * lane;
         const int4 e4 = ld4(w.E, base), s4 = ld4(w.SB, base), f4 = ld4(w.F, base);
@@ -594,6 +611,7 @@ __device__ __forceinline__ void derive_one(const Ws &w, int A, int tb, int &SB0,
 __device__ __forceinline__ void compact(const Ws &w, int &A, int tb) {
     const int lane = lane_id();
     int wpos = 0;
+    #pragma unroll 1
     for (int cb = 0; cb < A; cb += kChunk) {
         const int base = cb + 4 * lane;
         const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
@@ -701,6 +719,7 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
     // le >= 0: #{old E <= E_m} already found by the admission test
     const int cnt = (lane < K) ? (le >= 0 ? le : lane_prefix_count(A, [&](int i) { return w.E[i] <= ne; })) : INT_MAX;
     const int last = ((A - 1) / kChunk) * kChunk;
+    #pragma unroll 1
     for (int cb = last; A > 0 && cb >= 0; cb -= kChunk) {
         const int base = cb + 4 * lane;
         const int4 e4 = ld4(w.E, base), f4 = ld4(w.F, base), b4 = ld4(w.B, base);
@@ -709,6 +728,7 @@ __device__ __forceinline__ bool insert_window(const Ws &w, int &A, int K, int t,
         const int bb[4] = {b4.x, b4.y, b4.z, b4.w}, pp[4] = {p4.x, p4.y, p4.z, p4.w};
         const int ii[4] = {i4.x, i4.y, i4.z, i4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
         int sh[4] = {0, 0, 0, 0};
+        #pragma unroll 1
         for (int m = 0; m < K; ++m) {
             const int c = __shfl_sync(FULL, cnt, m);
 #pragma unroll
@@ -751,6 +771,7 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
     const unsigned ball = __ballot_sync(FULL, lane < W && need + incl > wint<N>(M));
     int phi = ball ? __ffs(ball) : W + 1;
     // active endpoints x = E_j >= t
+    #pragma unroll 1
     for (int j = lane; j < A; j += 32) {
         const int ej = w.E[j];
         if (ej < t) continue;
@@ -766,6 +787,7 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
         const wint<N> base = v0 - w.wcs[r] - wint<N>(r) * d;
         if (base + csW + wint<N>(W) * d <= wint<N>(M)) continue;
         int lo = r + 1, hi = W;
+        #pragma unroll 1
         while (lo < hi) {
             const int mid = (lo + hi) >> 1;
             if (base + w.wcs[mid] + wint<N>(mid) * d > wint<N>(M)) hi = mid; else lo = mid + 1;
@@ -781,6 +803,7 @@ __device__ __forceinline__ int admissible_prefix_search(const Ws &w, int A, int 
         const wint<N> base = av - ex - wint<N>(lane) * d;  // ex = CS[lane]
         if (base + csW + wint<N>(W) * d > wint<N>(M)) {
             int lo = lane + 1, hi = W;
+            #pragma unroll 1
             while (lo < hi) {
                 const int mid = (lo + hi) >> 1;
                 if (base + w.wcs[mid] + wint<N>(mid) * d > wint<N>(M)) hi = mid; else lo = mid + 1;
@@ -825,6 +848,7 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
         // by two binary searches in step
         const int y = t + dm;
         int lo1 = 0, hi1 = A, lo2 = 0, hi2 = A;
+        #pragma unroll 1
         while (lo1 < hi1 || lo2 < hi2) {
             const int m1 = (lo1 + hi1) >> 1, m2 = (lo2 + hi2) >> 1;
             const int e1 = w.E[min(m1, A - 1)], e2 = w.E[min(m2, A - 1)];
@@ -841,6 +865,7 @@ __device__ __forceinline__ int admissible_prefix(const Ws &w, int A, int tb, int
     }
     wint<N> need = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
     // two candidates per round: the state after both is used only if neither fails
+    #pragma unroll 1
     for (int k = 1; k <= W; k += 2) {
         const bool two = k < W;
         const int s1 = __shfl_sync(FULL, mine.s, k - 1) + 1;
@@ -884,6 +909,7 @@ __device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int
                                                          int W, const QEnt &mine) {
     const int lane = lane_id();
     const int Mi = int(M);
+    #pragma unroll 1
     for (int j = lane; j < A; j += 32) {
         const int ej = w.E[j];
         w.K[j] = (ej >= t) ? satw<N>(wint<N>(w.SB[j]) + wint<N>(A - j) * (wint<N>(ej) - tb)) : INT_MIN;
@@ -896,12 +922,14 @@ __device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int
         av = satw<N>(wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb));
     }
     wint<N> need = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
+    #pragma unroll 1
     for (int k = 1; k <= W; ++k) {
         const int c = k - 1;
         const int sc = __shfl_sync(FULL, mine.s, c) + 1;
         const int Lc = __shfl_sync(FULL, mine.key, c);
         need += sc;
         bool fail = false;
+        #pragma unroll 1
         for (int j = lane; j < A; j += 32) {  // each lane updates only its own points
             const int v = w.K[j];
             const int dj = w.E[j] - t;
@@ -923,6 +951,7 @@ __device__ __forceinline__ int admissible_prefix_general(const Ws &w, int A, int
 __device__ __forceinline__ void sort_admitted(const Ws &w, int K, QEnt &mine) {
     const int lane = lane_id();
     int rk = 0;
+    #pragma unroll 1
     for (int m = 0; m < K; ++m) {
         const int Lo = __shfl_sync(FULL, mine.key, m);
         rk += (Lo < mine.key || (Lo == mine.key && m < lane)) ? 1 : 0;
@@ -961,6 +990,7 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
     if (yup <= y0) return kBig;
     const W C = W(M) - s - L;  // (2): PM - C <= y;  (3): y <= floor((C - SB[j]) / (A - j))
     W best = BIG;
+    #pragma unroll 1
     for (int j = lane; j <= A; j += 32) {
         const W prev = (j == 0) ? -BIG : W(w.E[j - 1] - tb);
         const W cur = (j == A) ? BIG : W(w.E[j] - tb);
@@ -990,6 +1020,7 @@ __device__ bool state_ok(const Ws &w, const Queue &q, int A, int tb, int SB0, in
     const int lane = lane_id();
     bool bad = false;
     int fmin = INT_MAX;
+    #pragma unroll 1
     for (int i = lane; i < A; i += 32) {
         const int e = w.E[i];
         if (i + 1 < A && e > w.E[i + 1]) bad = true;
@@ -1001,9 +1032,11 @@ __device__ bool state_ok(const Ws &w, const Queue &q, int A, int tb, int SB0, in
         if ((POL == P_AMAX || POL == P_HSF || POL == P_AR) && w.F[i] > e) bad = true;
     }
     if (lane == 0 && (w.SB[A] != 0 || w.PM[0] != INT_MIN || (A > 0 && w.SB[0] != SB0))) bad = true;
+    #pragma unroll 1
     for (int i = lane; i + 1 < q.dn; i += 32)
         if (!qless(w.dq[i + 1], w.dq[i])) bad = true;
     if (q.mcb >= 0)
+        #pragma unroll 1
         for (int i = q.mh + lane; i + 1 < min(q.me, q.mcb + kMc); i += 32)
             if (i >= q.mcb && !qless(w.mc[i - q.mcb], w.mc[i + 1 - q.mcb])) bad = true;
     fmin = __reduce_min_sync(FULL, fmin);
@@ -1129,6 +1162,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         if (POL == P_AMIN) {
             wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
             if (need > wint<N>(M)) {
+                #pragma unroll 1
                 while (need > wint<N>(M)) {
                     int pos;
                     if (kib >= 0) {
@@ -1152,6 +1186,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                             bp = (best == mk && mk != UINT_MAX) ? base + j : -1;
                             pos = int(__reduce_min_sync(FULL, bp >= 0 ? unsigned(bp) : UINT_MAX));
                         } else {
+                        #pragma unroll 1
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
                             const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
@@ -1174,6 +1209,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     } else {
                         unsigned bk = UINT_MAX, bi = UINT_MAX;
                         int bp = -1;
+                        #pragma unroll 1
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
                             const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
@@ -1227,6 +1263,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 break;
             }
             const int c = warp_prefix_count(A, [&](int i) { return w.E[i] < t; });
+            #pragma unroll 1
             for (int j = 0; j < c; ++j) {  // in position order; the delta orders equal keys by index
                 const int b = w.B[j], p = w.P[j], f = w.F[j], id = w.I[j];
                 QEnt e;
@@ -1263,6 +1300,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     prefix_le_lt(w.E, A, y, hi, lb);
                 } else {
                     lb = hi;
+                    #pragma unroll 1
                     while (hi < A && w.E[hi] <= y) ++hi;
                 }
                 pdirty = false;
