@@ -387,6 +387,22 @@ __device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &
     const int lane = lane_id();
     if (q.dn == w.dcap) merge_delta(w, q);
     const int dn = q.dn;
+    if (dn < 64) {
+        // two entries per lane: count the entries greater than e (they lead the descending delta),
+        // then the smaller ones move one place right straight from registers
+        QEnt d0, d1;
+        const bool h0 = lane < dn, h1 = lane + 32 < dn;
+        if (h0) d0 = w.dq[lane];
+        if (h1) d1 = w.dq[lane + 32];
+        const int pos = __popc(__ballot_sync(FULL, h0 && qless(e, d0))) + __popc(__ballot_sync(FULL, h1 && qless(e, d1)));
+        __syncwarp();
+        if (h0 && lane >= pos) w.dq[lane + 1] = d0;
+        if (h1 && lane + 32 >= pos) w.dq[lane + 33] = d1;
+        if (lane == 0) w.dq[pos] = e;
+        __syncwarp();
+        q.dn = dn + 1;
+        return;
+    }
     const int pos = warp_prefix_count(dn, [&](int i) { return qless(e, w.dq[i]); });  // #entries > e
     #pragma unroll 1
     for (int hi = dn; hi > pos; hi -= 32) {
