@@ -1178,30 +1178,34 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         if (POL == P_AMIN) {
             wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
             if (need > wint<N>(M)) {
+                // one-chunk sets with packed keys: the keys stay in registers for all of the step's
+                // cancellations; a cancelled key becomes UINT_MAX
+                const bool reg = kib >= 0 && A <= kChunk;
+                unsigned key[4] = {UINT_MAX, UINT_MAX, UINT_MAX, UINT_MAX};
+                if (reg) {
+                    const int base = 4 * lane;
+                    const int4 k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                    const int kk[4] = {k4.x, k4.y, k4.z, k4.w}, ii[4] = {i4.x, i4.y, i4.z, i4.w};
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        key[j] = (base + j < A) ? (unsigned(kk[j]) << kib) | unsigned(ii[j]) : UINT_MAX;
+                }
                 #pragma unroll 1
                 while (need > wint<N>(M)) {
                     int pos;
-                    if (kib >= 0) {
+                    if (reg) {
+                        // a min tree over this lane's four keys, then the position
+                        const unsigned best = min(min(key[0], key[1]), min(key[2], key[3]));
+                        const unsigned mk = __reduce_min_sync(FULL, best);
+                        const int j = key[0] == mk ? 0 : (key[1] == mk ? 1 : (key[2] == mk ? 2 : 3));
+                        const bool own = best == mk && mk != UINT_MAX;
+                        pos = int(__reduce_min_sync(FULL, own ? unsigned(4 * lane + j) : UINT_MAX));
+#pragma unroll
+                        for (int m = 0; m < 4; ++m) key[m] = (own && m == j) ? UINT_MAX : key[m];
+                    } else if (kib >= 0) {
                         // (estimate, index) packed into one 32-bit key: one reduction for the minimum
                         unsigned best = UINT_MAX;
                         int bp = -1;
-                        if (A <= kChunk) {
-                            // one chunk: a min tree over this lane's four keys, then the position
-                            const int base = 4 * lane;
-                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
-                            const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
-                            unsigned key[4];
-#pragma unroll
-                            for (int j = 0; j < 4; ++j)
-                                key[j] = (base + j < A && ff[j] >= 0) ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
-                                                                     : UINT_MAX;
-                            best = min(min(key[0], key[1]), min(key[2], key[3]));
-                            const unsigned mk = __reduce_min_sync(FULL, best);
-                            const int j = key[0] == mk ? 0 : (key[1] == mk ? 1 : (key[2] == mk ? 2 : 3));
-                            bp = (best == mk && mk != UINT_MAX) ? base + j : -1;
-                            pos = int(__reduce_min_sync(FULL, bp >= 0 ? unsigned(bp) : UINT_MAX));
-                        } else {
                         #pragma unroll 1
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
@@ -1210,18 +1214,17 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                             const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
-                                const unsigned key = (base + j < A && ff[j] >= 0)
-                                                         ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
-                                                         : UINT_MAX;
-                                if (key < best) {
-                                    best = key;
+                                const unsigned kj = (base + j < A && ff[j] >= 0)
+                                                        ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
+                                                        : UINT_MAX;
+                                if (kj < best) {
+                                    best = kj;
                                     bp = base + j;
                                 }
                             }
                         }
                         const unsigned mk = __reduce_min_sync(FULL, best);
                         pos = int(__reduce_min_sync(FULL, (bp >= 0 && best == mk) ? unsigned(bp) : UINT_MAX));
-                        }
                     } else {
                         unsigned bk = UINT_MAX, bi = UINT_MAX;
                         int bp = -1;
