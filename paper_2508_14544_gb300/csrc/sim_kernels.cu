@@ -467,9 +467,9 @@ __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *ru
     }
 }
 
-// First kWin entries of R_t in (key, idx) order, by a merge path over the cached head of the main
-// array (ascending) and the delta (descending): lane m finds how many of the m smallest entries
-// come from the main array and returns entry m in `mine` (src 0 main, 1 delta).  Returns how many.
+// First kWin entries of R_t in (key, idx) order from the cached head of the main array (ascending)
+// and the delta (descending): lane m returns entry m in `mine` (src 0 main, 1 delta).  Returns how
+// many there are.
 __device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, int &msrc) {
     const int lane = lane_id();
     const int nmain = max(q.me - q.mh, 0);
@@ -477,21 +477,43 @@ __device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, i
     const int na = min(kWin, nmain);
     const int dn = q.dn;
     const int nb = min(kWin, dn);
-    const QEnt *A = w.mc + (q.mh - q.mcb);  // A[i], ascending
-    const QEnt *Bd = w.dq + (dn - 1);       // B[j] = Bd[-j], ascending
-    int lo = max(0, lane - nb), hi = min(lane, na);
-    #pragma unroll 1
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (qless(A[mid], Bd[-(lane - 1 - mid)])) lo = mid + 1; else hi = mid;
+    // The main head A (ascending, lane i holds A[i]) followed by the delta head B in descending
+    // order (lane i holds B[31 - i]) is a bitonic sequence of 64; the lane-wise minimum of the two
+    // halves holds the 32 smallest entries of both as a bitonic sequence, which five shuffle stages
+    // sort.  Missing entries are +infinity (key and index INT_MAX, above every real entry).  With one
+    // source empty the other's head, read in ascending order, is the window as it stands.
+    QEnt x;
+    x.key = x.idx = INT_MAX;
+    x.s = x.o = 0;
+    int src = 0;
+    if (lane < na) x = w.mc[q.mh - q.mcb + lane];
+    const int jb = (na > 0) ? kWin - 1 - lane : lane;  // one source only: its head is the window
+    if (jb < nb) {
+        const QEnt y = w.dq[dn - 1 - jb];
+        if (qless(y, x)) {
+            x = y;
+            src = 1;
+        }
     }
-    const int j = lane - lo;
+#pragma unroll
+    for (int d = 16; na > 0 && nb > 0 && d >= 1; d >>= 1) {
+        QEnt y;
+        y.key = __shfl_xor_sync(FULL, x.key, d);
+        y.idx = __shfl_xor_sync(FULL, x.idx, d);
+        y.s = __shfl_xor_sync(FULL, x.s, d);
+        y.o = __shfl_xor_sync(FULL, x.o, d);
+        const int ysrc = __shfl_xor_sync(FULL, src, d);
+        const bool lower = (lane & d) == 0;
+        if (lower == qless(y, x)) {  // the lower lane keeps the smaller entry
+            x = y;
+            src = ysrc;
+        }
+    }
     const int W = min(kWin, na + nb);
     msrc = 0;
     if (lane < W) {
-        const bool take_a = j >= nb || (lo < na && qless(A[lo], Bd[-j]));
-        mine = take_a ? A[lo] : Bd[-j];
-        msrc = take_a ? 0 : 1;
+        mine = x;
+        msrc = src;
     }
     return W;
 }
