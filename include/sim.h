@@ -130,9 +130,10 @@ int sim_create(int policy, int64_t M, int32_t n_instances, sim_ctx **out);
  *              simulation itself to know when a job finishes).
  *   device_ptrs 0: the arrays are host memory; 1: device memory on the current device, already
  *               written (the call does not order itself after the caller's streams).
- * The library copies the data into device buffers it owns (on a stream of its own, so the call
- * does not wait for other work on the device); the caller may free or reuse its arrays as soon as
- * the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
+ * The library stages the data into device buffers it owns (host arrays are copied in first; device
+ * arrays are read in place by the staging kernel), on a stream of its own, so the call does not
+ * wait for other work on the device, and returns when staging has finished: the caller may free
+ * or reuse its arrays as soon as the call returns.  Per-instance input problems (INVAL, INFEASIBLE) do not fail
  * the call: they are reported in that instance's sim_result.status by sim_run.
  * Returns SIM_OK, SIM_E_INVAL (n_per_instance < 0, null pointer; under SIM_AR, which needs
  * sim_load_ranked_csr), SIM_E_NOMEM or SIM_E_CUDA.

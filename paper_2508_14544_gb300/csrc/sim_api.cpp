@@ -62,6 +62,7 @@ struct sim_ctx {
     size_t main_bytes = 0;
     double *d_cr = nullptr;
     cudaStream_t load_stream = nullptr;  // non-blocking stream of sim_load (independent of other threads' work)
+    int64_t *h_off = nullptr;            // pinned copy of the offsets (n_inst + 1) for their upload
     int64_t launches = 0;
     std::vector<DevResult> h_res;
     std::string err;
@@ -226,15 +227,28 @@ static int load_impl(sim_ctx *c, const int64_t *offsets, const int32_t *a, const
     if (!c->load_stream && (e = cudaStreamCreateWithFlags(&c->load_stream, cudaStreamNonBlocking)) != cudaSuccess)
         return cuda_fail(c, e, "sim_load: stream creation");
     const cudaStream_t ls = c->load_stream;
-    const cudaMemcpyKind kind = device_ptrs ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    // Device inputs are read in place by the staging kernel (sim_load returns only after it has
+    // finished, so the caller may reuse them afterwards); host inputs are copied in first.
     const int32_t *src[6] = {a, s, l, u, o, rank};
     const int nsrc = (c->policy == SIM_AR) ? 6 : 5;
+    const int32_t *in[6];
+    for (int k = 0; k < 6; ++k) in[k] = c->d_raw + size_t(k) * c->cap_total;
     for (int k = 0; k < nsrc; ++k) {
         if (nt == 0) break;
-        e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t), kind, ls);
+        if (device_ptrs) {
+            in[k] = src[k];
+            continue;
+        }
+        e = cudaMemcpyAsync(c->d_raw + size_t(k) * c->cap_total, src[k], size_t(nt) * sizeof(int32_t),
+                            cudaMemcpyHostToDevice, ls);
         if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the input arrays");
     }
-    e = cudaMemcpyAsync(c->d_off, offsets, size_t(c->n_inst + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, ls);
+    if (!c->h_off && (e = cudaMallocHost(&c->h_off, size_t(c->n_inst + 1) * sizeof(int64_t))) != cudaSuccess) {
+        c->h_off = nullptr;
+        return cuda_fail(c, e, "sim_load: pinned offsets buffer");
+    }
+    std::memcpy(c->h_off, offsets, size_t(c->n_inst + 1) * sizeof(int64_t));
+    e = cudaMemcpyAsync(c->d_off, c->h_off, size_t(c->n_inst + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, ls);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_load: copy of the offsets");
     simgb::StageParams sp;
     sp.policy = c->policy;
@@ -243,12 +257,12 @@ static int load_impl(sim_ctx *c, const int64_t *offsets, const int32_t *a, const
     sp.n_max = int32_t(n_max);
     sp.step_cap = c->step_cap;
     sp.off = c->d_off;
-    sp.a = c->d_raw;
-    sp.s = c->d_raw + c->cap_total;
-    sp.l = c->d_raw + 2 * c->cap_total;
-    sp.u = c->d_raw + 3 * c->cap_total;
-    sp.o = c->d_raw + 4 * c->cap_total;
-    sp.rank = c->d_raw + 5 * c->cap_total;
+    sp.a = in[0];
+    sp.s = in[1];
+    sp.l = in[2];
+    sp.u = in[3];
+    sp.o = in[4];
+    sp.rank = in[5];
     sp.lu = c->d_lu;
     sp.rec = c->d_rec;
     sp.rec_a = c->d_rec_a;
@@ -515,6 +529,7 @@ void sim_destroy(sim_ctx *c) {
     dfree(c->d_main);
     dfree(c->d_cr);
     if (c->load_stream) cudaStreamDestroy(c->load_stream);
+    if (c->h_off) cudaFreeHost(c->h_off);
     delete c;
 }
 
