@@ -228,6 +228,34 @@ def test_long_requests_narrow_and_wide_kernels_agree():
             assert np.array_equal(wide[f], ref[f]), (pol, f)
 
 
+def test_cancellation_order_without_packed_keys():
+    """A_min packs (estimate, index) into one 32-bit key when the instance's longest length and its
+    request count fit.  Here 4096 requests (12 index bits) and upper bounds of 1.2e6 (21 bits) do
+    not, so cancellations use the two-level (estimate, index) comparison; an instance of 1000
+    requests with short lengths next to it takes the packed path.  Both kernels equal the oracle."""
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(33)
+    parts = []
+    for n, big in ((4096, True), (1000, False)):
+        o = rng.integers(1, 40, n)
+        l = np.maximum(o // 4, 1)
+        u = o * 4
+        if big:
+            u[rng.choice(n, 3, replace=False)] = 1_200_000
+        s = rng.integers(1, 8, n)
+        parts.append(dict(a=np.zeros(n, np.int64), s=s, l=l, u=u, o=o))
+    w = W.concat_instances("unpacked", 600, parts)
+    for pol in (1, 2):
+        ref = oracle_run(pol, w)
+        narrow, _ = gpu_run(pol, w)
+        wide, _ = gpu_run(pol, w, debug_checks=1)
+        for f in FIELDS:
+            assert np.array_equal(narrow[f], ref[f]), (pol, f)
+            assert np.array_equal(wide[f], ref[f]), (pol, f)
+        if pol == 1:
+            assert ref["evictions"][0] > 100 and ref["evictions"][1] > 100
+
+
 def test_command_lines(capsys):
     """`python -m paper_2508_14544_gb300.run` and `.sweep` through the C ABI."""
     import json
