@@ -1149,9 +1149,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     int tb_next = 0;
     for (;;) {
         if (pend_compact) {
-            // jobs marked dead (cancelled or completed) leave the active set.  Both kinds of
-            // removal share this one site: the loop body stays small, which matters when two
-            // warps at different points of it share a scheduler's instruction cache.
+            // cancelled jobs (F = -1) and jobs completed at the previous step (F = tb - 1) leave
+            // the active set.  Both kinds of removal share this one site: the loop body stays
+            // small, which matters when two warps at different points of it share a scheduler's
+            // instruction cache.
             tb = tb_next;
             const int A0 = A;
             compact_derive<N>(w, A, tb, SB0, nextF);
