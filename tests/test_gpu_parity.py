@@ -62,6 +62,43 @@ def test_random_tiny_batch(pol, arrivals):
     assert np.array_equal(comp, rcomp)
 
 
+def _random_mixed_workload(seed, M):
+    """Instance sizes around the kernel's size thresholds (delta capacity 64 / 128 / 256 at 1024 /
+    4096 requests, one-chunk active sets up to 128 jobs, windows of 32), random accuracy, memory
+    limits from tight to loose, and arrivals at t=0, spread out, or in bursts."""
+    from fractions import Fraction
+
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(seed)
+    parts = []
+    sizes = [1, 7, 31, 33, 63, 65, 200, 1000, 1024, 1025, 2100, 4096, 4097]
+    for i in range(2 * len(sizes)):
+        n = sizes[i % len(sizes)]
+        s = rng.integers(1, 17, n)
+        o = rng.integers(1, 61, n)
+        alpha = [Fraction(1, 10), Fraction(1, 4), Fraction(1, 2), Fraction(1)][i % 4]
+        l, u = W.interval_for(o, alpha, rng)
+        kind = (i // len(sizes) + i) % 3
+        if kind == 0:
+            a = np.zeros(n, np.int64)
+        elif kind == 1:
+            a = np.sort(rng.integers(0, 3 * n + 1, n))
+        else:
+            a = np.sort(rng.integers(0, 8, n)) * 250
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    return W.concat_instances("mixed", M, parts)
+
+
+@pytest.mark.parametrize("M", [700, 6000])
+@pytest.mark.parametrize("pol", POLS)
+def test_random_mixed_sizes(pol, M):
+    w = _random_mixed_workload(7, M)
+    got, comp = gpu_run(pol, w, completions=True)
+    ref, rcomp = oracle_run(pol, w, completions=True)
+    assert_same(got, ref, tag=f"mixed pol={pol}")
+    assert np.array_equal(comp, rcomp)
+
+
 @pytest.mark.parametrize("pol", POLS)
 def test_c1(pol):
     from paper_2508_14544_gb300 import workloads as W
