@@ -33,14 +33,24 @@ Readings of the text that this oracle fixes (each is also listed in the design n
   for A_max and H-SF), so if S' alone fails at some future step nothing is admitted.
 * Admission order.  The eligible waiting set (arrived, not active, not done) is sorted by
   (key, request index) with key = u (A_max), õ (A_min) or o (H-SF); the policy admits the largest
-  feasible *prefix* ("in order", Algorithm milb).  The papers' "break ties uniformly at random"
-  becomes "smaller request index first"; the workload generator makes index order random.
+  feasible *prefix* ("in order", Algorithm milb).  The paper's "break ties uniformly at random"
+  becomes "smaller request index first": the workload generator draws the requests i.i.d., so
+  the index order of requests that have not yet run is a uniformly random order that the policy
+  has observed nothing about, and a fixed random order of such requests admits the same
+  subsets, in law, as a fresh draw every step.
 * A_min eviction (Algorithm milb / milbrevise).  If sum_{i in S_t} (s_i + g_i + 1) > M, sort S_t by
-  (õ_i, index) ascending and remove jobs one at a time until the rest fits.  Each removed job:
-  eviction count + 1, õ_i <- max(õ_i, g_i) (the refinement never lowers a certified lower bound),
-  g_i <- 0, back to the waiting set, and eligible in the same step's admission ("unprocessed or
-  restartable requests", Section 4).  Both the max and the same-step eligibility are switchable
-  for sensitivity studies (``refine`` / ``same_step``).
+  õ_i ascending, ties "uniformly at random", and remove jobs one at a time until the rest fits.
+  The random tie order is drawn afresh at every step: job i's tie key at step t is
+  ``tie_key(seed, t, i)``, a counter-based draw (SplitMix64, below), and S_t is sorted by
+  (õ_i, tie key, index).  The seed is an input (one per instance), so runs are reproducible.
+  A fixed order such as the request index would not be a fair draw here: admission also takes
+  ties in index order, so among active jobs of equal õ the lowest index started first and has
+  generated the most tokens, and an index rule would always cancel the most advanced of them.
+  Each removed job: eviction count + 1, õ_i <- max(õ_i, g_i) (the refinement never lowers a
+  certified lower bound), g_i <- 0, back to the waiting set, and eligible in the same step's
+  admission ("unprocessed or restartable requests", Section 4).  The max, the same-step
+  eligibility and the tie rule are switchable for sensitivity studies (``refine``, ``same_step``,
+  ``evict_ties="index"`` for the index order).
 * A_r (Algorithm random, Appendix B).  The true lengths o, and a fixed random permutation given as
   ``rank`` (rank[i] = position of request i; the draw is an input, not made here).  Admission is
   the largest feasible prefix of the waiting set in (rank, index) order, as for the other
@@ -74,6 +84,28 @@ OK, E_INVAL, E_INFEASIBLE, E_STEPCAP = 0, -1, -2, -3
 _WAITING, _ACTIVE, _DONE = 0, 1, 2
 
 
+_MASK64 = (1 << 64) - 1
+
+
+def splitmix64(seed: int, k: int) -> int:
+    """Output number k (k >= 1) of the SplitMix64 generator seeded with ``seed`` (Steele, Lea and
+    Flood, "Fast splittable pseudorandom number generators", OOPSLA 2014, with the finalizer of
+    Vigna's public-domain splitmix64.c): the state after k steps is seed + k * 0x9E3779B97F4A7C15
+    (mod 2^64), and the output is that state passed through two xor-shift-multiply rounds and a
+    final xor-shift."""
+    z = (seed + k * 0x9E3779B97F4A7C15) & _MASK64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _MASK64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _MASK64
+    return z ^ (z >> 31)
+
+
+def tie_key(seed: int, t: int, i: int) -> int:
+    """Random tie key of request i at step t for A_min's eviction order: the high 32 bits of
+    SplitMix64 output number (t * 2^32 + i) + 1.  One counter per (step, request), so every step
+    draws a fresh, independent order of the tied jobs."""
+    return splitmix64(seed & _MASK64, ((t << 32) | i) + 1) >> 32
+
+
 def default_step_cap(o: Sequence[int]) -> int:
     return 64 * (len(o) + sum(int(x) for x in o))
 
@@ -103,13 +135,21 @@ def _empty_result(status: int, n: int) -> dict:
 
 def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
              refine: str = "max", same_step: bool = True, trace: list | None = None,
-             rank: Sequence[int] | None = None) -> dict:
+             rank: Sequence[int] | None = None, tie_seed: int = 0, evict_ties: str = "hash",
+             admit_ties: str = "index") -> dict:
     """Run one instance; return the result record plus per-request completion steps.
 
     ``trace`` (optional list) receives one dict per processed step: t, the batch, the admitted
     and the evicted (A_min) or promoted (A_ell) request indices, and the step's memory.
     ``rank`` is A_r's permutation (rank[i] = position of request i), required for A_r only.
+    ``tie_seed`` seeds A_min's random eviction ties (``evict_ties="hash"``, the paper's rule);
+    ``evict_ties="index"`` breaks them by request index instead (sensitivity studies only).
+    ``admit_ties="hash"`` (sensitivity studies only) orders the waiting set by (key, fresh random
+    draw, index) at every step, the draw being ``tie_key(~tie_seed, t, i)``, instead of by
+    (key, index).
     """
+    if evict_ties not in ("hash", "index") or admit_ties not in ("hash", "index"):
+        raise ValueError((evict_ties, admit_ties))
     n = len(o)
     a = [int(x) for x in a]
     s = [int(x) for x in s]
@@ -186,7 +226,10 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
         if policy == AMIN:
             need = sum(s[i] + gen[i] + 1 for i in active)
             if need > M:
-                order = sorted(active, key=lambda i: (otil[i], i))
+                if evict_ties == "hash":
+                    order = sorted(active, key=lambda i: (otil[i], tie_key(tie_seed, t, i), i))
+                else:
+                    order = sorted(active, key=lambda i: (otil[i], i))
                 for i in order:
                     if need <= M:
                         break
@@ -220,7 +263,10 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
                 active = [i for i in active if state[i] == _ACTIVE]
                 waiting = waiting + evicted
 
-        waiting.sort(key=lambda i: (key(i), i))
+        if admit_ties == "hash":
+            waiting.sort(key=lambda i: (key(i), tie_key(~tie_seed & _MASK64, t, i), i))
+        else:
+            waiting.sort(key=lambda i: (key(i), i))
         admitted = []
         for i in waiting:
             if feasible(active, admitted + [i]):

@@ -10,7 +10,9 @@
  * (Section 3.1) with the policy's length estimate (o for H-SF, Algorithm off; u for A_max,
  * Algorithm malb; the running lower bound for A_min, Algorithms milb / milbrevise), admission of
  * the largest feasible prefix of the waiting set sorted by (key, index), and A_min's
- * overflow eviction in ascending (lower bound, index) order with the refinement
+ * overflow eviction in ascending lower-bound order, ties broken by a random key drawn afresh at
+ * every step (SplitMix64 of the instance's seed and the counter step * 2^32 + index; the index
+ * order instead when evict_index is set), with the refinement
  * lower_bound <- max(lower_bound, tokens generated).  A_r (Algorithm random): true lengths and a
  * given permutation rank as the queue key.  A_ell (Algorithm promote_l): FIFO queue (key 2 a_i on
  * arrival, 2 t + 1 on re-entry at step t), estimate l_i, and at the start of a step a request that
@@ -114,14 +116,33 @@ static int validate(int policy, int64_t M, int32_t n, const int32_t *a, const in
     return O_OK;
 }
 
+/* ---- A_min's random eviction ties ---------------------------------------------------------------
+ * SplitMix64 (Steele, Lea and Flood, OOPSLA 2014; finalizer of Vigna's public-domain splitmix64.c):
+ * output number k >= 1 for a seed is the state seed + k * 0x9E3779B97F4A7C15 (mod 2^64) passed
+ * through two xor-shift-multiply rounds and a final xor-shift.  The tie key of request i at step t
+ * is the high half of output number (t * 2^32 + i) + 1. */
+static uint64_t splitmix64_at(uint64_t seed, uint64_t k) {
+    uint64_t z = seed + k * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+uint32_t oracle_tie_key(uint64_t seed, int64_t t, int32_t i) {
+    const uint64_t k = (((uint64_t)t << 32) | (uint32_t)i) + 1u;
+    return (uint32_t)(splitmix64_at(seed, k) >> 32);
+}
+
 typedef struct {
     int32_t key, idx;
+    uint32_t tie; /* random tie key (0 for every job under the index rule) */
     int64_t w;
 } evk_t;
 
 static int cmp_evk(const void *pa, const void *pb) {
     const evk_t *a = (const evk_t *)pa, *b = (const evk_t *)pb;
     if (a->key != b->key) return (a->key > b->key) - (a->key < b->key);
+    if (a->tie != b->tie) return (a->tie > b->tie) - (a->tie < b->tie);
     return (a->idx > b->idx) - (a->idx < b->idx);
 }
 
@@ -145,10 +166,12 @@ int64_t oracle_default_step_cap(int32_t n, const int32_t *o) {
  * Simulate one instance.  step_cap <= 0 selects the default cap 64 * (n + sum o).
  * completion (optional, n entries) receives each request's completion step C_i.
  * rank (A_r only; may be NULL otherwise) is the permutation position of each request.
+ * tie_seed seeds A_min's random eviction ties; evict_index != 0 breaks them by index instead.
  */
-int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
-                  const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
-                  int64_t step_cap, oracle_result *res, int64_t *completion) {
+int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+                      const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                      uint64_t tie_seed, int evict_index, int64_t step_cap, oracle_result *res,
+                      int64_t *completion) {
     memset(res, 0, sizeof(*res));
     if (completion)
         for (int32_t i = 0; i < n; i++) completion[i] = 0;
@@ -214,7 +237,7 @@ int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int3
             continue;
         }
 
-        /* A_min: overflow of the next step -> evict in ascending (lower bound, index) */
+        /* A_min: overflow of the next step -> evict in ascending (lower bound, tie key, index) */
         if (policy == O_AMIN) {
             int64_t need = 0;
             for (int32_t k = 0; k < an; k++) need += s[act[k]] + (t - start[act[k]]) + 1;
@@ -223,6 +246,7 @@ int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int3
                     int32_t i = act[k];
                     ev[k].key = otil[i];
                     ev[k].idx = i;
+                    ev[k].tie = evict_index ? 0u : oracle_tie_key(tie_seed, t, i);
                     ev[k].w = s[i] + (t - start[i]) + 1;
                 }
                 qsort(ev, (size_t)an, sizeof(evk_t), cmp_evk);
@@ -326,6 +350,12 @@ int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int3
     return status;
 }
 
+int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+                  const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                  int64_t step_cap, oracle_result *res, int64_t *completion) {
+    return oracle_run_seeded(policy, M, n, a, s, l, u, o, rank, 0, 0, step_cap, res, completion);
+}
+
 int oracle_run(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
                const int32_t *l, const int32_t *u, const int32_t *o, int64_t step_cap,
                oracle_result *res, int64_t *completion) {
@@ -339,6 +369,8 @@ typedef struct {
     int32_t n_inst;
     const int64_t *off;
     const int32_t *a, *s, *l, *u, *o, *rank;
+    const uint64_t *tie_seed;
+    int evict_index;
     int64_t step_cap;
     oracle_result *res;
     int64_t *completion;
@@ -354,23 +386,28 @@ static void *batch_worker(void *arg) {
         pthread_mutex_unlock(&b->mu);
         if (i >= b->n_inst) break;
         int64_t lo = b->off[i], hi = b->off[i + 1];
-        oracle_run_ex(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
-                      b->u + lo, b->o + lo, b->rank ? b->rank + lo : NULL, b->step_cap, &b->res[i],
-                      b->completion ? b->completion + lo : NULL);
+        oracle_run_seeded(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
+                          b->u + lo, b->o + lo, b->rank ? b->rank + lo : NULL,
+                          b->tie_seed ? b->tie_seed[i] : 0, b->evict_index, b->step_cap, &b->res[i],
+                          b->completion ? b->completion + lo : NULL);
     }
     return NULL;
 }
 
-int oracle_run_batch_ex(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
-                        const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
-                        const int32_t *o, const int32_t *rank, int64_t step_cap, oracle_result *res,
-                        int64_t *completion, int32_t n_threads) {
+/* Many instances (CSR offsets); tie_seed (optional, one per instance, else 0 for all). */
+int oracle_run_batch_seeded(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                            const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                            const int32_t *o, const int32_t *rank, const uint64_t *tie_seed,
+                            int evict_index, int64_t step_cap, oracle_result *res,
+                            int64_t *completion, int32_t n_threads) {
     batch_t b;
     b.policy = policy;
     b.M = M;
     b.n_inst = n_inst;
     b.off = offsets;
     b.a = a; b.s = s; b.l = l; b.u = u; b.o = o; b.rank = rank;
+    b.tie_seed = tie_seed;
+    b.evict_index = evict_index;
     b.step_cap = step_cap;
     b.res = res;
     b.completion = completion;
@@ -389,6 +426,14 @@ int oracle_run_batch_ex(int policy, int64_t M, int32_t n_inst, const int64_t *of
     for (int32_t i = 0; i < n_inst; i++)
         if (res[i].status < worst) worst = res[i].status;
     return worst;
+}
+
+int oracle_run_batch_ex(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                        const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                        const int32_t *o, const int32_t *rank, int64_t step_cap, oracle_result *res,
+                        int64_t *completion, int32_t n_threads) {
+    return oracle_run_batch_seeded(policy, M, n_inst, offsets, a, s, l, u, o, rank, NULL, 0,
+                                   step_cap, res, completion, n_threads);
 }
 
 int oracle_run_batch(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,

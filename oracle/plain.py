@@ -58,6 +58,17 @@ def lib():
                                           i32p, i32p, i32p, i32p, ctypes.c_int64, ctypes.c_void_p, i64p,
                                           ctypes.c_int32]
         L.oracle_run_batch_ex.restype = ctypes.c_int
+        u64p = ctypes.POINTER(ctypes.c_uint64)
+        L.oracle_run_seeded.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i32p, i32p, i32p, i32p,
+                                        i32p, i32p, ctypes.c_uint64, ctypes.c_int, ctypes.c_int64,
+                                        ctypes.c_void_p, i64p]
+        L.oracle_run_seeded.restype = ctypes.c_int
+        L.oracle_run_batch_seeded.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, i64p, i32p, i32p,
+                                              i32p, i32p, i32p, i32p, u64p, ctypes.c_int, ctypes.c_int64,
+                                              ctypes.c_void_p, i64p, ctypes.c_int32]
+        L.oracle_run_batch_seeded.restype = ctypes.c_int
+        L.oracle_tie_key.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int32]
+        L.oracle_tie_key.restype = ctypes.c_uint32
         L.oracle_default_step_cap.argtypes = [ctypes.c_int32, i32p]
         L.oracle_default_step_cap.restype = ctypes.c_int64
         _lib = L
@@ -80,17 +91,30 @@ def _p64(x: np.ndarray | None):
     return x.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
 
 
+def _evict_index(evict_ties: str) -> int:
+    if evict_ties not in ("hash", "index"):
+        raise ValueError(evict_ties)
+    return 1 if evict_ties == "index" else 0
+
+
+def tie_key(seed: int, t: int, i: int) -> int:
+    """A_min's random tie key of request i at step t (the C oracle's own SplitMix64)."""
+    return int(lib().oracle_tie_key(int(seed) & ((1 << 64) - 1), int(t), int(i)))
+
+
 def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool = False,
-        rank=None) -> dict:
+        rank=None, tie_seed: int = 0, evict_ties: str = "hash") -> dict:
     """One instance.  Returns the result fields (and 'completion' if asked).  ``rank`` is A_r's
-    permutation (rank[i] = position of request i)."""
+    permutation (rank[i] = position of request i); ``tie_seed`` seeds A_min's random eviction
+    ties (``evict_ties="index"``: by request index instead)."""
     a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
     rank = None if rank is None else _i32(rank)
     n = int(o.shape[0])
     res = np.zeros(1, dtype=RESULT_DTYPE)
     comp = np.zeros(max(n, 1), dtype=np.int64) if completions else None
-    lib().oracle_run_ex(int(policy), int(M), n, _p32(a), _p32(s), _p32(l), _p32(u), _p32(o), _p32(rank),
-                        int(step_cap), res.ctypes.data, _p64(comp))
+    lib().oracle_run_seeded(int(policy), int(M), n, _p32(a), _p32(s), _p32(l), _p32(u), _p32(o), _p32(rank),
+                            int(tie_seed) & ((1 << 64) - 1), _evict_index(evict_ties), int(step_cap),
+                            res.ctypes.data, _p64(comp))
     out = {k: int(res[0][k]) for k in FIELDS}
     if completions:
         out["completion"] = comp[:n].tolist()
@@ -98,28 +122,36 @@ def run(policy: int, M: int, a, s, l, u, o, step_cap: int = 0, completions: bool
 
 
 def run_batch(policy: int, M: int, offsets, a, s, l, u, o, step_cap: int = 0, n_threads: int = 1,
-              completions: bool = False, rank=None):
+              completions: bool = False, rank=None, tie_seeds=None, evict_ties: str = "hash"):
     """Many instances in CSR layout.  Returns a structured array (RESULT_DTYPE) and optionally the
-    per-request completion steps."""
+    per-request completion steps.  ``tie_seeds``: one uint64 per instance (default 0 for all)."""
     offsets = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
     a, s, l, u, o = (_i32(v) for v in (a, s, l, u, o))
     rank = None if rank is None else _i32(rank)
     n_inst = int(offsets.shape[0] - 1)
+    seeds = None
+    if tie_seeds is not None:
+        seeds = np.ascontiguousarray(np.asarray(tie_seeds, dtype=np.uint64))
+        assert seeds.shape == (n_inst,)
     res = np.zeros(n_inst, dtype=RESULT_DTYPE)
     comp = np.zeros(max(int(offsets[-1]), 1), dtype=np.int64) if completions else None
-    lib().oracle_run_batch_ex(int(policy), int(M), n_inst, _p64(offsets), _p32(a), _p32(s), _p32(l),
-                              _p32(u), _p32(o), _p32(rank), int(step_cap), res.ctypes.data, _p64(comp),
-                              int(n_threads))
+    sp = ctypes.POINTER(ctypes.c_uint64)() if seeds is None else seeds.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64))
+    lib().oracle_run_batch_seeded(int(policy), int(M), n_inst, _p64(offsets), _p32(a), _p32(s), _p32(l),
+                                  _p32(u), _p32(o), _p32(rank), sp, _evict_index(evict_ties), int(step_cap),
+                                  res.ctypes.data, _p64(comp), int(n_threads))
     if completions:
         return res, comp[: int(offsets[-1])]
     return res
 
 
-def run_workload(policy: int, w, step_cap: int = 0, n_threads: int = 1, completions: bool = False):
-    """Convenience: run a ``Workload`` (from the seeded generator) through the C oracle."""
+def run_workload(policy: int, w, step_cap: int = 0, n_threads: int = 1, completions: bool = False,
+                 evict_ties: str = "hash"):
+    """Convenience: run a ``Workload`` (from the seeded generator) through the C oracle, with the
+    workload's own A_min tie seeds."""
     return run_batch(policy, w.M, w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o,
                      step_cap=step_cap, n_threads=n_threads, completions=completions,
-                     rank=w.ranks() if policy == 3 else None)
+                     rank=w.ranks() if policy == 3 else None, tie_seeds=w.tie_seeds(),
+                     evict_ties=evict_ties)
 
 
 def default_step_cap(o) -> int:

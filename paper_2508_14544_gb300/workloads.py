@@ -21,6 +21,10 @@ in the fixed order s, o, l, arrivals, so any subset of instances is reproducible
 The auxiliary policy A_r (Algorithm random) also needs a uniformly random permutation of each
 instance's requests; ``Workload.ranks()`` draws it from a separate stream,
 ``numpy.random.default_rng([seed0 + i, 1])``, and returns rank[j] = position of request j.
+
+A_min breaks eviction ties uniformly at random (Algorithm milb).  The simulator and the oracle
+draw those ties themselves from a counter-based generator; the generator only supplies its seed,
+one uint64 per instance: ``Workload.tie_seeds()`` = seed0 + i.
 """
 from __future__ import annotations
 
@@ -98,6 +102,14 @@ class Workload:
                 out[lo:hi] = rk
             self._ranks = out
         return self._ranks
+
+    def tie_seeds(self) -> np.ndarray:
+        """Seed of A_min's random eviction ties for every instance (uint64): seed0 + id (instance
+        id = global id when known, else the row)."""
+        base = 0 if self.seed0 is None else int(self.seed0)
+        ids = np.arange(self.n_instances, dtype=np.int64) if self.instance_ids is None else \
+            np.asarray(self.instance_ids, dtype=np.int64)
+        return (ids + base).astype(np.uint64)
 
     def uniform_n(self) -> int | None:
         d = np.diff(self.offsets)

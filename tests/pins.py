@@ -96,7 +96,19 @@ def aell_wave_cases():
     return out
 
 
-def check_all(sim) -> list:
+def tie_vectors():
+    """(seed, k, expected high 32 bits of SplitMix64 output k) from the published vectors."""
+    out = []
+    for v in load("splitmix64.json")["vectors"]:
+        outs = [int(x, 16) for x in v["outputs_hex"]] if "outputs_hex" in v else [int(x) for x in v["outputs"]]
+        for k, z in enumerate(outs, start=1):
+            out.append((int(v["seed"]), k, z >> 32))
+    return out
+
+
+def check_all(sim, tie_key=None) -> list:
+    """Run every pin against ``sim``; ``tie_key(seed, t, i)`` (optional) is checked against the
+    published SplitMix64 vectors and the tie keys listed in the hand traces."""
     fails = []
 
     def chk(tag, got, exp):
@@ -109,12 +121,23 @@ def check_all(sim) -> list:
             elif got.get(key) != val:
                 fails.append((tag, key, got.get(key), val))
 
-    def run(tag, *args, rank=None):
+    def run(tag, *args, rank=None, tie_seed=None):
+        kw = {}
+        if rank is not None:
+            kw["rank"] = rank
+        if tie_seed is not None:
+            kw["tie_seed"] = tie_seed
         try:
-            return sim(*args, rank=rank) if rank is not None else sim(*args)
+            return sim(*args, **kw)
         except AssertionError as e:  # an internal invariant tripped
             fails.append((tag, "assertion", str(e), None))
             return None
+
+    if tie_key is not None:
+        for seed, k, hi in tie_vectors():
+            got = tie_key(seed, 0, k - 1)
+            if got != hi:
+                fails.append((f"splitmix64/{seed}/{k}", "tie_key", got, hi))
 
     pe = load("paper_examples.json")
     ex = pe["example1"]
@@ -132,9 +155,15 @@ def check_all(sim) -> list:
         if name.startswith("_"):
             continue
         r = run(name, POL[case["policy"]], case["M"], case["a"], case["s"], case["l"], case["u"], case["o"],
-                rank=case.get("rank"))
+                rank=case.get("rank"), tie_seed=case.get("tie_seed"))
         if r is not None:
             chk(name, r, case["expect"])
+        if tie_key is not None and "tie_keys" in case:
+            for t, keys in case["tie_keys"].items():
+                for i, want in enumerate(keys):
+                    got = tie_key(case["tie_seed"], int(t), i)
+                    if got != want:
+                        fails.append((name, f"tie_key({t},{i})", got, want))
 
     for tag, M, a, s, l, u, o, exp in wave_cases():
         for p in (AMAX, AMIN, HSF):

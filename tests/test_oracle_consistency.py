@@ -27,8 +27,8 @@ def test_literal_equals_plain_random():
     for trial in range(400):
         M, a, s, l, u, o = _rand_case(rng, arrivals=bool(trial % 2))
         for p in (0, 1, 2):
-            r1 = literal.simulate(p, M, a, s, l, u, o)
-            r2 = plain.run(p, M, a, s, l, u, o, completions=True)
+            r1 = literal.simulate(p, M, a, s, l, u, o, tie_seed=trial)
+            r2 = plain.run(p, M, a, s, l, u, o, completions=True, tie_seed=trial)
             assert _same(r1, r2), (p, M, a.tolist(), s.tolist(), l.tolist(), u.tolist(), o.tolist())
 
 
@@ -111,8 +111,10 @@ def test_plain_batch_matches_single():
     w = W.make_workload("c2", [0, 300, 600, 900])
     for p in (0, 1, 2):
         rb = plain.run_workload(p, w, n_threads=4)
+        seeds = w.tie_seeds()
         for i in range(w.n_instances):
             inst = w.instance(i)
-            r = plain.run(p, inst["M"], inst["a"], inst["s"], inst["l"], inst["u"], inst["o"])
+            r = plain.run(p, inst["M"], inst["a"], inst["s"], inst["l"], inst["u"], inst["o"],
+                          tie_seed=int(seeds[i]))
             for f in pins.FIELDS + ("status",):
                 assert int(rb[i][f]) == r[f]

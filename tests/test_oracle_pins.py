@@ -6,14 +6,17 @@ from oracle import literal, plain
 from tests import pins
 
 SIMS = {
-    "literal": lambda p, M, a, s, l, u, o, rank=None: literal.simulate(p, M, a, s, l, u, o, rank=rank),
-    "plain": lambda p, M, a, s, l, u, o, rank=None: plain.run(p, M, a, s, l, u, o, completions=True, rank=rank),
+    "literal": lambda p, M, a, s, l, u, o, rank=None, tie_seed=0: literal.simulate(p, M, a, s, l, u, o, rank=rank,
+                                                                                  tie_seed=tie_seed),
+    "plain": lambda p, M, a, s, l, u, o, rank=None, tie_seed=0: plain.run(p, M, a, s, l, u, o, completions=True,
+                                                                          rank=rank, tie_seed=tie_seed),
 }
+TIE_KEYS = {"literal": literal.tie_key, "plain": plain.tie_key}
 
 
 @pytest.mark.parametrize("which", sorted(SIMS))
 def test_all_pins(which):
-    fails = pins.check_all(SIMS[which])
+    fails = pins.check_all(SIMS[which], tie_key=TIE_KEYS[which])
     assert not fails, fails
 
 
