@@ -1,19 +1,23 @@
 #!/usr/bin/env python3
 """Throughput of the batched scheduler simulator on one GB300 (or N, one replica per GPU).
 
-One step = one pass of the whole path over the 1024-instance workload (1024 instances x 1000
-requests, all arriving at t=0, M=16384, s~U{1..64}, o~U{1..512}, alpha in {1/5,1/2,4/5,1}):
-for each of A_max, A_min and H-SF, load the (device-resident) request arrays through sim_load
-(staging: validation + sort of the waiting set) and simulate every instance with sim_run; then
-compute the competitive ratios TEL(A_max)/TEL(H-SF) and TEL(A_min)/TEL(H-SF).
+One step = one pass of the whole path over the alpha-sweep workload (alpha = 1/10 .. 10/10 x 4096
+seeds = 40960 instances x 2000 requests, all arriving at t=0, M=32768, s~U{16..256}, bimodal o:
+70% U{1..32}, 30% U{512..2048}), the largest of the five configurations: for each of A_max, A_min
+and H-SF, load the (device-resident) request arrays through sim_load (staging: validation + sort
+of the waiting set) and simulate every instance with sim_run; then compute the competitive ratios
+TEL(A_max)/TEL(H-SF) and TEL(A_min)/TEL(H-SF).
 
 The metric is simulated request-steps per second: the sum over instances and policies of
 sum_t |batch_t| (tokens generated, wasted A_min tokens included), divided by the device time.
+After the timed region the other four configurations are timed per policy (sub-records), the
+per-step method's work is counted (SIM_OPT_COUNT_WORK) for the roofline, whose integer-issue and
+shared-memory ceilings are measured on the GPU (sim_measure_peaks).
 
   python bench.py [--gpus N --steps K --warmup W]          # the CUDA path
   python bench.py --impl reference [...]                     # the CPU oracle on a bounded sample
-Under torchrun each rank simulates its own 1024 instances (weak scaling; no collective on the
-data path: instances are independent); rank 0 prints one JSON line.
+Under torchrun each rank simulates its own copy of the workload's shape (weak scaling; no
+collective on the data path: instances are independent); rank 0 prints one JSON line.
 """
 from __future__ import annotations
 
@@ -33,25 +37,34 @@ sys.path.insert(0, str(ROOT))
 
 METRIC = "simulated request-steps/s (A_min, A_max)"
 UNIT = "request-steps/s"
-WORKLOAD = "c2"
-WORKLOAD_DESC = ("1024 instances x n=1000 requests at t=0, M=16384, s~U{1..64}, o~U{1..512}, "
-                 "alpha in {1/5,1/2,4/5,1} (256 seeds each); policies A_max, A_min, H-SF + CR")
+WORKLOAD = "c4"
+WORKLOAD_DESC = ("alpha in {1/10..10/10} x 4096 seeds = 40960 instances x n=2000 requests at t=0, M=32768, "
+                 "s~U{16..256}, o: 70% U{1..32}, 30% U{512..2048}; policies A_max, A_min, H-SF + CR")
+SUB_WORKLOADS = ("c1", "c2", "c3", "c5")
 POLICY_NAMES = ("A_max", "A_min", "H-SF")
-# Algorithmic work model of one request-step (one token of one batch member): tokens += 1,
-# compare with the true length, add to the step's memory and to the request-step count.
-OPS_PER_REQUEST_STEP = 4
-INT32_LANES_PER_SM = 128
+
+# Work of the paper's per-step method (Theorem complexity) per unit, for the roofline:
+#   per request-step (one token of one batch member): 4 int ops (tokens + 1, compare with the true
+#     length, add to the step's memory and to the request-step count), 8 bytes of shared memory;
+#   per S2 add (memory accounting of the active set): 1 int op;
+#   per S3 compare-exchange (sorting the active set on an overflow): 3 int ops, 8 bytes;
+#   per S5 endpoint evaluation (binary-searched admission): 6 int ops, 16 bytes;
+#   per S4 queue operation (one insert and one removal per admission): 1 int op, 16 bytes each;
+#   global memory: the 20-byte request once, the 56-byte result, and the bytes the waiting queue
+#     moves (counted by the kernel).
+OPS = {"request_step": 4, "s2": 1, "s3": 3, "s5": 6, "s4": 1}
+SMEM_B = {"request_step": 8, "s3": 8, "s5": 16, "s4": 16}
 
 
 def _dram_traffic(kernel: str) -> int | None:
-    """DRAM bytes per launch of `kernel` on this workload, from the committed ncu summary, or None
-    when the simulation kernel's sources changed since those counters were taken."""
+    """DRAM bytes per launch of `kernel` on the bench workload, from the committed ncu summary, or
+    None when the simulation kernel's sources changed since those counters were taken."""
     import hashlib
     p = ROOT / "profiles" / "dram_traffic.json"
     if not p.exists():
         return None
     entry = json.loads(p.read_text()).get(kernel)
-    if not entry:
+    if not entry or entry.get("workload_key") != WORKLOAD:
         return None
     h = hashlib.sha256()
     for f in entry["sources"]:
@@ -121,51 +134,51 @@ def dist_env():
     return rank, world, local
 
 
-def make_rank_workload(rank: int):
+def make_rank_workload(rank: int, name: str = WORKLOAD):
     from paper_2508_14544_gb300 import workloads as W
-    return W.make_workload(WORKLOAD, W.rank_instances(WORKLOAD, rank))
+    return W.make_workload(name, W.rank_instances(name, rank))
 
 
-def cpu_baseline(w, max_seconds: float = 20.0) -> dict:
-    """The CPU oracle as it stands, on the whole workload once per policy, all host cores.
-
-    One pass of the three policies over every instance is ~1.6 s of wall time on 16 Arm cores
-    (about 25 CPU-seconds); later policies are skipped if the budget of max_seconds runs out."""
+def cpu_baseline(w, budget_s: float = 20.0) -> dict:
+    """The CPU oracle as it stands (oracle/plain.c, all host cores, one instance per task) on a
+    bounded sample of the workload: every k-th instance, all three policies, k chosen from a
+    first timed pass so that the whole sample takes about budget_s of wall time."""
     from oracle import plain
     cores = os.cpu_count() or 1
+    first = w.subset(range(0, w.n_instances, 320))  # 128 instances, all alphas
+    t0 = time.perf_counter()
+    for pol in (0, 1, 2):
+        plain.run_workload(pol, first, n_threads=cores)
+    per_inst = (time.perf_counter() - t0) / first.n_instances
+    stride = max(1, int(w.n_instances / max(1.0, budget_s / max(per_inst, 1e-6))))
+    sample = w.subset(range(0, w.n_instances, stride))
     rs = 0
     t0 = time.perf_counter()
     c0 = time.process_time()
-    done = 0
     for pol in (0, 1, 2):
-        r = plain.run_workload(pol, w, n_threads=cores)
-        rs += int(r["request_steps"].sum())
-        done += 1
-        if time.perf_counter() - t0 > max_seconds:
-            break
+        rs += int(plain.run_workload(pol, sample, n_threads=cores)["request_steps"].sum())
     dt = time.perf_counter() - t0
     cpu_s = time.process_time() - c0
     return {"value": rs / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"all {w.n_instances} instances x {done} policies (A_max, A_min, H-SF), "
-                      f"oracle/plain.c with {cores} threads: {dt:.1f} s wall, {cpu_s:.1f} CPU-s"}
+            "sample": f"every {stride}th instance ({sample.n_instances} of {w.n_instances}, all alphas) x 3 policies "
+                      f"(A_max, A_min, H-SF), oracle/plain.c with {cores} threads: {dt:.1f} s wall, {cpu_s:.1f} CPU-s"}
 
 
 def run_reference(args) -> None:
     rank, world, local = dist_env()
     if rank != 0:
         return
-    w = make_rank_workload(0)
-    t_all = []
-    rs_all = 0
     from oracle import plain
+    from paper_2508_14544_gb300 import workloads as W
     cores = os.cpu_count() or 1
-    sample = w.subset(range(0, w.n_instances, 4))
+    n_all = W.WORKLOADS[WORKLOAD].n_instances
+    sample = W.make_workload(WORKLOAD, range(0, n_all, 320))  # 128 instances per step, all alphas
+    t_all, rs_all = [], 0
     for it in range(args.warmup + args.steps):
         t0 = time.perf_counter()
         rs = 0
         for pol in (0, 1, 2):
-            r = plain.run_workload(pol, sample, n_threads=cores)
-            rs += int(r["request_steps"].sum())
+            rs += int(plain.run_workload(pol, sample, n_threads=cores)["request_steps"].sum())
         dt = time.perf_counter() - t0
         if it >= args.warmup:
             t_all.append(dt)
@@ -176,11 +189,103 @@ def run_reference(args) -> None:
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / max(args.steps, 1),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD_DESC, "sample": f"{sample.n_instances} instances (every 4th)"},
+            "config": {"workload": WORKLOAD_DESC, "sample": f"{sample.n_instances} instances (every 320th) per step"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"{sample.n_instances} of {w.n_instances} instances x 3 policies per step"},
+                             "sample": f"{sample.n_instances} of {n_all} instances x 3 policies per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def _time_runs(sim, stream, load_args, reps: int, with_load: bool = True):
+    """(median sim_load ms, median sim_run ms, last results) by CUDA events on the stream."""
+    import torch
+    lm, rm, res = [], [], None
+    for _ in range(reps):
+        e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        torch.cuda.synchronize()
+        e0.record(stream)
+        if with_load:
+            sim.load(*load_args)
+        e1.record(stream)
+        res = sim.run(stream.cuda_stream)
+        e2.record(stream)
+        torch.cuda.synchronize()
+        lm.append(e0.elapsed_time(e1))
+        rm.append(e1.elapsed_time(e2))
+    return statistics.median(lm), statistics.median(rm), res
+
+
+def algorithmic_work(res, wc, n_requests: int) -> dict:
+    """Per-launch work of the per-step method from the results and the kernel's work counters."""
+    rs = int(res["request_steps"].sum())
+    ev = int(res["evictions"].sum())
+    s2, s3, s5, gq = (int(x) for x in wc.sum(axis=0))
+    s4 = 2 * (n_requests + ev)
+    ops = OPS["request_step"] * rs + OPS["s2"] * s2 + OPS["s3"] * s3 + OPS["s5"] * s5 + OPS["s4"] * s4
+    smem = SMEM_B["request_step"] * rs + SMEM_B["s3"] * s3 + SMEM_B["s5"] * s5 + SMEM_B["s4"] * s4
+    hbm = 20 * n_requests + 56 * len(res) + gq
+    return {"request_steps": rs, "s2_adds": s2, "s3_compare_exchanges": s3, "s5_endpoint_evals": s5,
+            "s4_queue_ops": s4, "queue_global_bytes": gq, "int_ops": ops, "smem_bytes": smem, "hbm_bytes": hbm}
+
+
+def sub_record(name: str, dev_id, stream, peaks_live: dict) -> dict:
+    """One of the other configurations: per policy sim_load and sim_run device time (median of 3
+    after a warm-up), request-steps/s, the dominant kernel; on the 10^5-request workload also the
+    global-memory rate of the per-step method's queue traffic."""
+    import torch
+
+    from paper_2508_14544_gb300 import SIM_AMAX, SIM_AMIN, SIM_HSF, Simulator
+    w = make_rank_workload(0, name)
+    d_in = [torch.from_numpy(np.ascontiguousarray(x)).to(dev_id) for x in
+            (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
+    rec = {"instances": w.n_instances, "requests": w.n_total}
+    per = {}
+    for pname, pol in zip(POLICY_NAMES, (SIM_AMAX, SIM_AMIN, SIM_HSF)):
+        with Simulator(pol, w.M, w.n_instances, tune_residency=1) as sim:
+            sim.set_tie_seeds(w.tie_seeds())
+            sim.load(w.offsets, *d_in)
+            r = sim.run(stream.cuda_stream)  # warm-up (and residency tuning)
+            assert np.all(r["status"] == 0), (name, pname, int(r["status"].min()))
+            lms, rms, r = _time_runs(sim, stream, (w.offsets, *d_in), 3)
+            rs = int(r["request_steps"].sum())
+            p = {"sim_load_ms": round(lms, 3), "sim_run_ms": round(rms, 3), "request_steps": rs,
+                 "request_steps_per_s": rs / (rms / 1000.0)}
+            if name == "c5":
+                sim.set_option("count_work", 1)
+                r2 = sim.run(stream.cuda_stream)
+                wk = algorithmic_work(r2, sim.work_counts(), w.n_total)
+                p["hbm_bytes_per_launch"] = wk["hbm_bytes"]
+                p["hbm_GBps"] = round(wk["hbm_bytes"] / (rms / 1000.0) / 1e9, 2)
+            per[pname] = p
+    dom = max(per, key=lambda k: per[k]["sim_run_ms"])
+    step_ms = sum(v["sim_load_ms"] + v["sim_run_ms"] for v in per.values())
+    rec.update({"policies": per, "dominant_kernel": f"k_run<{dom}>",
+                "request_steps_per_s": sum(v["request_steps"] for v in per.values()) / (step_ms / 1000.0)})
+    if name == "c5":
+        gb = per[dom]["hbm_GBps"]
+        rec["hbm_of_measured"] = round(gb / float(_peaks().get("hbm_gbs", 6800.0)), 5)
+    return rec
+
+
+def critical_path_c2(dev_id, stream) -> dict:
+    """A_min on the 1024-instance workload: the launch time against its slowest instance alone."""
+    import torch
+
+    from paper_2508_14544_gb300 import SIM_AMIN, Simulator
+    w = make_rank_workload(0, "c2")
+    with Simulator(SIM_AMIN, w.M, w.n_instances, tune_residency=1) as sim:
+        sim.load_workload(w)
+        r = sim.run(stream.cuda_stream)
+        _, full_ms, r = _time_runs(sim, stream, None, 3, with_load=False)
+    slow = int(np.argmax(r["evictions"]))
+    one = w.subset([slow])
+    with Simulator(SIM_AMIN, one.M, 1) as sim:
+        sim.load_workload(one)
+        sim.run(stream.cuda_stream)
+        _, alone_ms, _ = _time_runs(sim, stream, None, 3, with_load=False)
+    return {"workload": "c2 (1024 x n=1000)", "policy": "A_min", "launch_ms": round(full_ms, 3),
+            "slowest_instance": slow, "its_cancellations": int(r["evictions"][slow]),
+            "alone_ms": round(alone_ms, 3), "launch_over_alone": round(full_ms / alone_ms, 3)}
 
 
 def run_ours(args) -> None:
@@ -189,7 +294,8 @@ def run_ours(args) -> None:
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2508_14544_gb300 import SIM_AELL, SIM_AMAX, SIM_AMIN, SIM_AR, SIM_HSF, Simulator
+    from paper_2508_14544_gb300 import SIM_AELL, SIM_AMAX, SIM_AMIN, SIM_AR, SIM_HSF, Simulator, cr_amin_lemma
+    from paper_2508_14544_gb300 import _lib as L
 
     rank, world, local = dist_env()
     if world > 1:
@@ -198,6 +304,7 @@ def run_ours(args) -> None:
     dev = torch.device("cuda", local)
     stream = torch.cuda.Stream(device=dev)
     sh = stream.cuda_stream
+    peaks_live = L.measure_peaks()
 
     w = make_rank_workload(rank)
     host = [np.ascontiguousarray(x) for x in (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
@@ -207,7 +314,8 @@ def run_ours(args) -> None:
     # each policy: a launch is as long as its slowest instance, and which residency is faster
     # depends on how uneven the instances are
     sims = [Simulator(p, w.M, w.n_instances, tune_residency=1) for p in (SIM_AMAX, SIM_AMIN, SIM_HSF)]
-    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
+    for s in sims:
+        s.set_tie_seeds(w.tie_seeds())
     torch.cuda.synchronize()
 
     def step(inputs):
@@ -219,35 +327,31 @@ def run_ours(args) -> None:
         return res, cr
 
     # warm-up (also checks that every instance finished)
-    for _ in range(max(args.warmup, 0)):
-        res, _ = step(d_in)
+    for _ in range(max(args.warmup, 1)):
+        res, cr = step(d_in)
     for r in res:
         assert np.all(r["status"] == 0), r["status"]
     rs_per_step = int(sum(int(r["request_steps"].sum()) for r in res))
     launches0 = sum(s.kernel_launches() for s in sims)
 
-    # timed region: K steps, device time by CUDA events on the simulator's stream
+    # timed region: K steps, device time by CUDA events on the simulator's stream; the inputs
+    # (1.6 GB per policy) are larger than the 129 MB L2, so no flush is needed between steps
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    load_starts = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    run_starts = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    run_ends = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(3)] for _ in range(args.steps)]
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
         time.sleep(0.3)
         for k in range(args.steps):
-            with torch.cuda.stream(stream):
-                flush.fill_(k & 0xff)
-            torch.cuda.synchronize()
             starts[k].record(stream)
             for j, sim in enumerate(sims):
-                load_starts[k][j].record(stream)
+                ev[k][j][0].record(stream)
                 sim.load(w.offsets, *d_in)
-                run_starts[k][j].record(stream)
+                ev[k][j][1].record(stream)
                 res[j] = sim.run(sh)
-                run_ends[k][j].record(stream)
+                ev[k][j][2].record(stream)
             sims[0].competitive_ratio(sims[2], sh)
             sims[1].competitive_ratio(sims[2], sh)
             ends[k].record(stream)
@@ -257,8 +361,8 @@ def run_ours(args) -> None:
     torch.cuda.synchronize()
     launches = sum(s.kernel_launches() for s in sims) - launches0
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    run_ms = [[run_starts[k][j].elapsed_time(run_ends[k][j]) for j in range(3)] for k in range(args.steps)]
-    load_ms = [[load_starts[k][j].elapsed_time(run_starts[k][j]) for j in range(3)] for k in range(args.steps)]
+    run_ms = [[ev[k][j][1].elapsed_time(ev[k][j][2]) for j in range(3)] for k in range(args.steps)]
+    load_ms = [[ev[k][j][0].elapsed_time(ev[k][j][1]) for j in range(3)] for k in range(args.steps)]
     total_s = sum(step_ms) / 1000.0
     if world > 1:
         t = torch.tensor([total_s], device=dev, dtype=torch.float64)
@@ -268,7 +372,7 @@ def run_ours(args) -> None:
 
     # end to end through the public API with host (pinned) buffers: H2D inside sim_load, D2H of
     # the per-instance results inside sim_run and of the ratios
-    e2e_steps = max(1, min(args.steps, 5))
+    e2e_steps = max(1, min(args.steps, 3))
     host_in = [p.numpy() for p in pinned]
     torch.cuda.synchronize()
     t0 = time.perf_counter()
@@ -281,10 +385,42 @@ def run_ours(args) -> None:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
     e2e_val = rs_per_step * e2e_steps * world / e2e_s
+    h2d = 3 * 5 * w.n_total * 4
+    d2h = 3 * w.n_instances * 56 + 2 * w.n_instances * 8
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    # ---- outside the timed region (rank 0) ----
+    # the per-step method's work in each policy's launch (SIM_OPT_COUNT_WORK; same results)
+    per_pol_ms = [statistics.mean(run_ms[k][j] for k in range(args.steps)) for j in range(3)]
+    work = []
+    for j, sim in enumerate(sims):
+        sim.set_option("count_work", 1)
+        r = sim.run(sh)
+        for f in ("total_latency", "request_steps", "evictions", "steps"):
+            assert np.array_equal(r[f], res[j][f]), f
+        work.append(algorithmic_work(r, sim.work_counts(), w.n_total))
+        sim.set_option("count_work", 0)
+    dom = int(np.argmax(per_pol_ms))
+    wd = work[dom]
+    sec = per_pol_ms[dom] / 1000.0
+    alu = {"achieved": wd["int_ops"] / sec / 1e12, "peak": peaks_live["int_ops_per_s"] / 1e12, "unit": "Tops/s"}
+    alu["frac"] = alu["achieved"] / alu["peak"]
+    smem = {"achieved": wd["smem_bytes"] / sec / 1e12, "peak": peaks_live["smem_bytes_per_s"] / 1e12, "unit": "TB/s"}
+    smem["frac"] = smem["achieved"] / smem["peak"]
+    hbm_peak = float(_peaks().get("hbm_gbs", 6800.0))
+    hbm = {"achieved": wd["hbm_bytes"] / sec / 1e9, "peak": hbm_peak, "unit": "GB/s",
+           "frac": wd["hbm_bytes"] / sec / 1e9 / hbm_peak}
+
+    # the other configurations, and the latency regime of the 1024-instance workload
+    subs = {name: sub_record(name, dev, stream, peaks_live) for name in SUB_WORKLOADS}
+    crit = critical_path_c2(dev, stream)
 
     # the paper's two further policies on the same instances (outside the step): A_r (Algorithm
-    # random, permutation drawn by the workload generator) and A_ell (Algorithm promote_l);
-    # sim_run device time by CUDA events, median of 3 after a warm-up
+    # random, permutation drawn by the workload generator) and A_ell (Algorithm promote_l)
     further = {}
     for name, pol in (("A_r", SIM_AR), ("A_ell", SIM_AELL)):
         with Simulator(pol, w.M, w.n_instances, tune_residency=1) as sim:
@@ -292,22 +428,12 @@ def run_ours(args) -> None:
             sim.load(w.offsets, *d_in, rank=rk)
             r = sim.run(sh)
             assert np.all(r["status"] == 0), (name, r["status"])
-            ms = []
-            for _ in range(3):
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                torch.cuda.synchronize()
-                e0.record(stream)
-                sim.run(sh)
-                e1.record(stream)
-                torch.cuda.synchronize()
-                ms.append(e0.elapsed_time(e1))
+            _, ms, r = _time_runs(sim, stream, None, 2, with_load=False)
         rsn = int(r["request_steps"].sum())
-        further[name] = {"sim_run_ms": round(statistics.median(ms), 3), "request_steps": rsn,
-                         "request_steps_per_s": rsn / (statistics.median(ms) / 1000.0)}
+        further[name] = {"sim_run_ms": round(ms, 3), "request_steps": rsn, "request_steps_per_s": rsn / (ms / 1000.0)}
 
     # the Lemma-thm:Amin evaluator on 2^20 histograms of 64 lengths (512 MB of doubles, read once):
     # 20 FP64 flops per length (6 FMA + 8 other), so GB300's FP64 rate bounds it, not HBM
-    from paper_2508_14544_gb300 import cr_amin_lemma
     hx = torch.rand((1 << 20, 64), dtype=torch.float64, device=dev)
     for _ in range(3):
         cr_amin_lemma(hx, 1, 0.0, stream=sh)
@@ -324,50 +450,48 @@ def run_ours(args) -> None:
     lemma_gbs = lemma_bytes / (statistics.median(lm) / 1000.0) / 1e9
     lemma_tflops = 20.0 * hx.numel() / (statistics.median(lm) / 1000.0) / 1e12
     del hx
-    h2d = 3 * 5 * w.n_total * 4
-    d2h = 3 * w.n_instances * 56 + 2 * w.n_instances * 8
 
-    if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
-        return
-    peaks = _peaks()
     clocks = clk.summary()
-    # roofline of the dominant kernel (the simulation kernel of the slowest policy): integer issue
-    per_pol_ms = [statistics.mean(run_ms[k][j] for k in range(args.steps)) for j in range(3)]
     rs_pol = [int(r["request_steps"].sum()) for r in res]
-    dom = int(np.argmax(per_pol_ms))
-    achieved_ops = OPS_PER_REQUEST_STEP * rs_pol[dom] / (per_pol_ms[dom] / 1000.0)
-    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    peak_ops = n_sm * INT32_LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": statistics.mean(step_ms), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
-        "config": {"workload": WORKLOAD_DESC, "instances_per_gpu": w.n_instances, "requests_per_instance": 1000,
+        "config": {"workload": WORKLOAD_DESC, "workload_key": WORKLOAD, "instances_per_gpu": w.n_instances,
+                   "requests_per_instance": 2000,
                    "parallelism": f"instances sharded, {world} replica(s), no collective on the data path",
-                   "l2": "256 MB buffer written between timed steps (inputs are 20 MB < L2)",
+                   "l2": "inputs larger than L2 (1.6 GB per policy against 129 MB); no flush",
                    "residency": "SIM_OPT_TUNE_RESIDENCY: one or two warps per scheduler, chosen per policy on the first warm-up run",
+                   "tie_seeds": "A_min cancellation ties: SplitMix64, seed 3000000 + instance id",
                    "request_steps_per_step": rs_per_step,
+                   "request_steps": dict(zip(POLICY_NAMES, rs_pol)),
                    "sim_run_ms": dict(zip(POLICY_NAMES, [round(x, 3) for x in per_pol_ms])),
                    "sim_load_ms": dict(zip(POLICY_NAMES, [round(statistics.mean(load_ms[k][j] for k in range(args.steps)), 3)
                                                           for j in range(3)])),
                    "batches_per_s": {POLICY_NAMES[j]: int(res[j]["steps"].sum()) / (per_pol_ms[j] / 1000.0)
                                      for j in range(3)},
-                   "us_per_instance": {POLICY_NAMES[j]: round(1000.0 * per_pol_ms[j] / w.n_instances, 3)
+                   "us_per_instance": {POLICY_NAMES[j]: round(1000.0 * per_pol_ms[j] / w.n_instances, 4)
                                        for j in range(3)},
+                   "mean_cr": {"A_max": float(np.nanmean(cr[0])), "A_min": float(np.nanmean(cr[1]))},
+                   "other_configs": subs,
+                   "critical_path": crit,
                    "further_policies_not_in_step": further,
                    "lemma_evaluator": {"histograms": 1 << 20, "lengths": 64, "ms": round(statistics.median(lm), 4),
                                        "GB_per_s": round(lemma_gbs, 1),
-                                       "frac_of_measured_hbm": round(lemma_gbs / float(_peaks().get("hbm_gbs", 6800.0)), 3),
+                                       "frac_of_measured_hbm": round(lemma_gbs / hbm_peak, 3),
                                        "fp64_tflops": round(lemma_tflops, 3),
                                        "frac_of_nominal_fp64_1.25": round(lemma_tflops / 1.25, 3)}},
         "roofline": {"bound": "alu", "kernel": f"k_run<{POLICY_NAMES[dom]}>",
-                     "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12,
-                     "unit": "Tops/s (int32)", "frac": achieved_ops / peak_ops,
+                     "achieved": alu["achieved"], "peak": alu["peak"], "unit": alu["unit"], "frac": alu["frac"],
                      "traffic": _dram_traffic(f"k_run<{POLICY_NAMES[dom]}>"),
-                     "model": f"{OPS_PER_REQUEST_STEP} int ops per request-step; peak = {n_sm} SMs x "
-                              f"{INT32_LANES_PER_SM} int32 lanes x {peaks.get('sm_max_mhz', 2070.0)} MHz"},
+                     "smem": smem, "hbm": hbm,
+                     "peaks": "measured live by sim_measure_peaks (integer issue: add/xor chains; shared memory: "
+                              "conflict-free 16-byte loads); HBM: MEASURED_PEAKS.json copy bandwidth",
+                     "work_per_launch": wd,
+                     "model": "work of the per-step method (Theorem complexity) counted by SIM_OPT_COUNT_WORK: "
+                              "4 ops/8 B per request-step, 1 op per S2 add, 3 ops/8 B per S3 compare-exchange, "
+                              "6 ops/16 B per S5 endpoint evaluation, 1 op/16 B per S4 queue operation; "
+                              "achieved = that work / the launch's CUDA-event time"},
         "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clocks,

@@ -11,7 +11,8 @@
  *              future step (eq. Constraint).  Never cancels a job.
  *   SIM_AMIN - A_min, Algorithms milb and milbrevise (Section 4, 4.2): each request starts with the
  *              lower bound l_i as its length estimate; when the next step would exceed M, active
- *              jobs are cancelled in ascending (estimate, index) order until the rest fits, and each
+ *              jobs are cancelled in ascending estimate order until the rest fits, ties broken
+ *              uniformly at random (a fresh draw at every step, see sim_set_tie_seeds), and each
  *              cancelled job's estimate becomes max(estimate, tokens generated); the waiting set is
  *              then admitted as for A_max, using the estimates.
  *   SIM_HSF  - the hindsight shortest-first benchmark H-SF, Algorithm off (Section 3.1, Appendix
@@ -32,9 +33,14 @@
  * (eq. constraintM).  Request i becomes eligible at step a_i (the paper has a_i = 0; arrivals are
  * an extension); its completion step C_i is one past the step that generated its last token.
  *
- * Ties that the paper breaks "uniformly at random" are broken by the smaller request index
- * (0-based position within the instance).  Outputs are deterministic and bit-identical to the CPU
- * reference of the same rules.
+ * Ties in the waiting set's order, which the paper breaks "uniformly at random", are broken by the
+ * smaller request index (0-based position within the instance): with requests drawn i.i.d. the
+ * index order of requests that have not run yet is itself a uniformly random order.  A_min's
+ * cancellation ties are drawn afresh at every step from a counter-based generator: the tie key of
+ * request i at step t is the high 32 bits of SplitMix64 output number t * 2^32 + i + 1 for the
+ * instance's seed (sim_set_tie_seeds), and the cancellation order is (estimate, tie key, index).
+ * Outputs are deterministic given the seeds and bit-identical to the CPU reference of the same
+ * rules.
  *
  * Threading: a context must not be used from two threads at once.  Different contexts are
  * independent.  All calls act on the CUDA device that is current on the calling thread.
@@ -95,7 +101,7 @@ enum {
                                        set, queue order; no job past its projected end under A_max,
                                        H-SF and A_r).  A violation gives that instance SIM_E_STATE.
                                        Slower; results are otherwise identical. */
-    SIM_OPT_TUNE_RESIDENCY = 7      /* 0/1: on the first sim_run of a load shape (n_instances, total
+    SIM_OPT_TUNE_RESIDENCY = 7,     /* 0/1: on the first sim_run of a load shape (n_instances, total
                                        and largest instance size), time the simulation launch with
                                        one warp per scheduler (4 per SM) and with the default
                                        residency, and use the faster for every later sim_run of
@@ -105,6 +111,13 @@ enum {
                                        cancellation chains), two when instances are even.  The
                                        tuning run simulates twice; results do not depend on it.
                                        Overrides SIM_OPT_WARPS_PER_SM while set. */
+    SIM_OPT_EVICT_TIES = 8,         /* 0 (default): A_min's cancellation ties are broken at random
+                                       as Algorithm milb states (see sim_set_tie_seeds); 1: by the
+                                       request index instead, a fixed order that always cancels the
+                                       earliest-started of the tied jobs (for sensitivity studies). */
+    SIM_OPT_COUNT_WORK = 9          /* 0/1: record per instance the work that the paper's per-step
+                                       method does (sim_get_work_counts; default 0).  Results are
+                                       identical; the counting costs a few instructions per event. */
 };
 
 /*
@@ -173,6 +186,38 @@ int sim_load_ranked_csr(sim_ctx *ctx, const int64_t *offsets, const int32_t *arr
 int sim_run(sim_ctx *ctx, sim_result *out, void *cuda_stream);
 
 /*
+ * sim_set_tie_seeds: seeds of A_min's random cancellation ties (Algorithm milb / milbrevise,
+ * Section 4: "sort S_t in ascending order of the lower bound; break ties uniformly at random").
+ *   seeds  HOST, n_instances uint64 values, one per instance; NULL resets every seed to 0 (the
+ *          default).  Copied before the call returns.
+ * At a step t with an overflow, the active jobs are cancelled in ascending (estimate, r, index)
+ * order, r = the high 32 bits of output number t * 2^32 + i + 1 of the SplitMix64 generator
+ * (Steele, Lea and Flood 2014) seeded with the instance's seed, i the request index: a fresh,
+ * reproducible random order of the tied jobs at every step.  Takes effect at the next sim_run (no
+ * reload needed); ignored under the other policies and under SIM_OPT_EVICT_TIES = 1.
+ * Returns SIM_OK, SIM_E_INVAL, SIM_E_STATE (another device is current), SIM_E_NOMEM or SIM_E_CUDA.
+ */
+int sim_set_tie_seeds(sim_ctx *ctx, const uint64_t *seeds);
+
+/*
+ * sim_get_work_counts: the work counters of the last sim_run (SIM_OPT_COUNT_WORK = 1), four int64
+ * per instance, instance-major, into `counts` (HOST, 4 * n_instances).  They count the work of
+ * the per-step method that Theorem complexity (Section 4) bounds, summed over the instance's
+ * processed steps, with A_t the active set at the start of step t, A'_t + k_t the batch after
+ * cancellations and admission (k_t admitted) and Q_t the waiting set at admission:
+ *   [0] sum_t A_t                                    (memory accounting of S_t: one add per job)
+ *   [1] sum over steps with an overflow (A_min) of A_t * ceil(log2 A_t)^2
+ *                                                    (compare-exchanges of a sort of S_t)
+ *   [2] sum_t (A'_t + k_t) * ceil(log2(Q_t + 1))     (endpoint evaluations of an admission that
+ *                                                     binary-searches the largest feasible prefix)
+ *   [3] bytes of global memory the waiting queue moved (arrival runs, head reloads, merges).
+ * The simulator itself skips most of this work (quiet steps in closed form, incremental order);
+ * the counters measure the method, not the kernel.  Returns SIM_OK, SIM_E_INVAL, SIM_E_STATE
+ * (counting was off for the last sim_run) or SIM_E_CUDA.
+ */
+int sim_get_work_counts(sim_ctx *ctx, int64_t *counts);
+
+/*
  * sim_get_completions: copy every request's completion step C_i of the last sim_run into
  * `completion_t` (HOST, n_total int64, same layout as the loaded arrays; 0 for instances that did
  * not run).  Requires SIM_OPT_RECORD_COMPLETIONS = 1 before sim_run; otherwise SIM_E_STATE.
@@ -209,7 +254,11 @@ int64_t sim_kernel_launches(const sim_ctx *ctx);
  * Everything except the inputs and outputs lives in one fixed array of about 23 MB that every GPU
  * loading the library holds until the process exits.  Limits: at most 2048 requests per instance
  * and 262,144 requests per call; larger inputs are rejected with SIM_E_INVAL and a message in
- * sim_last_error(NULL).  All calls share that array and it keeps the last call's contents: calls
+ * sim_last_error(NULL).  The staging kernel checks the offsets it reads against the same limits
+ * again: an instance that reaches past them gets status SIM_E_INVAL in its result and nothing of
+ * it is staged.  The fixed array holds the workspaces of 128 simulating warps (32 blocks of 4),
+ * so on a 152-SM GPU most SMs stay idle: with many instances expect several times the time of
+ * sim_run, which sizes its launch to the whole GPU.  All calls share that array and it keeps the last call's contents: calls
  * that overlap on the GPU (different streams or threads) race; calls on one stream are safe.
  * The first call on each device looks up the array's device address (cudaGetSymbolAddress) with
  * that device current; make that first call before any stream capture.  Allocates nothing.

@@ -19,6 +19,8 @@ SIM_OPT_STEP_CAP, SIM_OPT_RECORD_COMPLETIONS, SIM_OPT_WARPS_PER_BLOCK, SIM_OPT_S
 SIM_OPT_WARPS_PER_SM = 5
 SIM_OPT_DEBUG_CHECKS = 6
 SIM_OPT_TUNE_RESIDENCY = 7
+SIM_OPT_EVICT_TIES = 8
+SIM_OPT_COUNT_WORK = 9
 
 STATUS_NAMES = {0: "SIM_OK", -1: "SIM_E_INVAL", -2: "SIM_E_INFEASIBLE", -3: "SIM_E_STEPCAP", -4: "SIM_E_CUDA",
                 -5: "SIM_E_STATE", -6: "SIM_E_NOMEM"}
@@ -37,8 +39,8 @@ RESULT_DTYPE = np.dtype([
 assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
 
 EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_load_ranked_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
-           "sim_set_option", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc",
-           "sim_cr_amin_lemma", "sim_cr_amin_rho")
+           "sim_set_option", "sim_set_tie_seeds", "sim_get_work_counts", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc",
+           "sim_cr_amin_lemma", "sim_cr_amin_rho", "sim_measure_peaks")
 
 _lib = None
 
@@ -80,6 +82,10 @@ def lib() -> ctypes.CDLL:
     L.sim_competitive_ratio.restype = ctypes.c_int
     L.sim_set_option.argtypes = [vp, ctypes.c_int, ctypes.c_int64]
     L.sim_set_option.restype = ctypes.c_int
+    L.sim_set_tie_seeds.argtypes = [vp, vp]
+    L.sim_set_tie_seeds.restype = ctypes.c_int
+    L.sim_get_work_counts.argtypes = [vp, vp]
+    L.sim_get_work_counts.restype = ctypes.c_int
     L.sim_last_error.argtypes = [vp]
     L.sim_last_error.restype = ctypes.c_char_p
     L.sim_destroy.argtypes = [vp]
@@ -93,6 +99,8 @@ def lib() -> ctypes.CDLL:
     L.sim_cr_amin_lemma.restype = ctypes.c_int
     L.sim_cr_amin_rho.argtypes = [ctypes.c_int32, vp, vp]
     L.sim_cr_amin_rho.restype = ctypes.c_int
+    L.sim_measure_peaks.argtypes = [vp]
+    L.sim_measure_peaks.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -114,6 +122,14 @@ def sim_last_error(ctx) -> str:
 
 def sim_set_option(ctx, key: int, value: int) -> int:
     return lib().sim_set_option(ctx, int(key), int(value))
+
+
+def sim_set_tie_seeds(ctx, seeds) -> int:
+    """Seeds of A_min's random cancellation ties: one uint64 per instance (host), or None."""
+    if seeds is None:
+        return lib().sim_set_tie_seeds(ctx, None)
+    arr = np.ascontiguousarray(np.asarray(seeds, dtype=np.uint64))
+    return lib().sim_set_tie_seeds(ctx, arr.ctypes.data)
 
 
 def _ptr(x) -> int:
@@ -144,6 +160,11 @@ def sim_load_ranked_csr(ctx, offsets: np.ndarray, a, s, l, u, o, rank, device_pt
 def sim_run(ctx, out: np.ndarray, stream: int = 0) -> int:
     assert out.dtype == RESULT_DTYPE and out.flags.c_contiguous
     return lib().sim_run(ctx, out.ctypes.data, ctypes.c_void_p(stream or None))
+
+
+def sim_get_work_counts(ctx, out: np.ndarray) -> int:
+    assert out.dtype == np.int64 and out.flags.c_contiguous
+    return lib().sim_get_work_counts(ctx, out.ctypes.data)
 
 
 def sim_get_completions(ctx, out: np.ndarray) -> int:
@@ -203,3 +224,14 @@ def cr_amin_rho(u_values) -> np.ndarray:
     if rc != SIM_OK:
         raise SimError(rc, sim_last_error(None))
     return out
+
+
+def measure_peaks() -> dict:
+    """Measured integer-issue and shared-memory-read ceilings of the current device
+    (include/sim_peaks.h)."""
+    out = np.zeros(4, dtype=np.float64)
+    rc = lib().sim_measure_peaks(out.ctypes.data)
+    if rc != 0:
+        raise SimError(rc, "sim_measure_peaks failed")
+    return {"int_ops_per_s": float(out[0]), "smem_bytes_per_s": float(out[1]), "int_ms": float(out[2]),
+            "smem_ms": float(out[3])}

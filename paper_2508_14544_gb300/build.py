@@ -14,7 +14,7 @@ CSRC = PKG / "csrc"
 INCLUDE = ROOT / "include"
 BUILD = PKG / "_build"
 LIB = BUILD / "libsim.so"
-SOURCES = ["sim_kernels.cu", "sim_stage.cu", "sim_api.cpp", "sim_noalloc.cu", "sim_analytic.cu"]
+SOURCES = ["sim_kernels.cu", "sim_stage.cu", "sim_api.cpp", "sim_noalloc.cu", "sim_analytic.cu", "sim_peaks.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -29,7 +29,7 @@ def _stale() -> bool:
     if not LIB.exists():
         return True
     t = LIB.stat().st_mtime
-    deps = [CSRC / s for s in SOURCES] + [CSRC / "sim_internal.h", INCLUDE / "sim.h", Path(__file__)]
+    deps = [CSRC / s for s in SOURCES] + [CSRC / "sim_internal.h", Path(__file__)] + sorted(INCLUDE.glob("*.h"))
     return any(d.stat().st_mtime > t for d in deps)
 
 

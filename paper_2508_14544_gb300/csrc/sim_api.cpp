@@ -31,6 +31,8 @@ struct sim_ctx {
     int warps_per_sm = 0;
     int debug_checks = 0;
     int tune_residency = 0;
+    int evict_index = 0;
+    int count_work = 0;
     // residency chosen by SIM_OPT_TUNE_RESIDENCY for the load shape tuned_shape (n_inst, n_total,
     // n_max): warps per SM, or 0 for the default; tuned_shape[0] < 0 when not tuned
     int tuned_wps = 0;
@@ -61,6 +63,9 @@ struct sim_ctx {
     QEnt *d_main = nullptr;
     size_t main_bytes = 0;
     double *d_cr = nullptr;
+    uint64_t *d_seed = nullptr;          // A_min tie seeds (n_inst), null until sim_set_tie_seeds
+    int64_t *d_wc = nullptr;             // work counters, 4 per instance (SIM_OPT_COUNT_WORK)
+    bool wc_valid = false;
     cudaStream_t load_stream = nullptr;  // non-blocking stream of sim_load (independent of other threads' work)
     int64_t *h_off = nullptr;            // pinned copy of the offsets (n_inst + 1) for their upload
     int64_t launches = 0;
@@ -169,6 +174,13 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
             c->tune_residency = value ? 1 : 0;
             c->tuned_shape[0] = -1;
             return SIM_OK;
+        case SIM_OPT_EVICT_TIES:
+            if (value != 0 && value != 1) return fail(c, SIM_E_INVAL, "EVICT_TIES must be 0 (random) or 1 (index)");
+            c->evict_index = int(value);
+            return SIM_OK;
+        case SIM_OPT_COUNT_WORK:
+            c->count_work = value ? 1 : 0;
+            return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
             if (value < 128 || value > 4096 || value % 128)
                 return fail(c, SIM_E_INVAL, "SMEM_ACTIVE_CAP must be a multiple of 128 in [128, 4096]");
@@ -255,6 +267,8 @@ static int load_impl(sim_ctx *c, const int64_t *offsets, const int32_t *a, const
     sp.M = c->M;
     sp.n_inst = c->n_inst;
     sp.n_max = int32_t(n_max);
+    sp.max_total = c->cap_total;
+    sp.max_n = INT32_MAX;
     sp.step_cap = c->step_cap;
     sp.off = c->d_off;
     sp.a = in[0];
@@ -361,10 +375,13 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.res = c->d_res;
     p.completion = c->record_completions ? c->d_comp : nullptr;
     p.lu = c->d_lu;
+    p.tie_seed = c->d_seed;
+    p.work_count = c->count_work ? c->d_wc : nullptr;
     p.ca = ca;
     p.dcap = dcap;
     p.use_smem = smem ? 1 : 0;
     p.debug = c->debug_checks;
+    p.evict_index = c->evict_index;
     p.gws = c->d_gws;
     p.gws_stride = int64_t(per_warp);
     p.mainbuf = c->d_main;
@@ -391,6 +408,13 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
             return fail(c, SIM_E_NOMEM, "sim_run: completion buffer");
         if ((e = cudaMemsetAsync(c->d_comp, 0, size_t(std::max<int64_t>(c->n_total, 1)) * sizeof(int64_t), st)) !=
             cudaSuccess)
+            return cuda_fail(c, e, "cudaMemsetAsync");
+    }
+    c->wc_valid = false;
+    if (c->count_work) {
+        if (!c->d_wc && (e = dalloc(c->d_wc, size_t(c->n_inst) * 4 * sizeof(int64_t))) != cudaSuccess)
+            return fail(c, SIM_E_NOMEM, "sim_run: work-counter buffer");
+        if ((e = cudaMemsetAsync(c->d_wc, 0, size_t(c->n_inst) * 4 * sizeof(int64_t), st)) != cudaSuccess)
             return cuda_fail(c, e, "cudaMemsetAsync");
     }
     // with SIM_OPT_DEBUG_CHECKS every instance runs in the checking global-memory kernel
@@ -464,6 +488,7 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
     }
     c->ran = true;
     c->comp_valid = c->record_completions != 0;
+    c->wc_valid = c->count_work != 0;
     if (worst == SIM_E_STATE) fail(c, SIM_E_STATE, "sim_run: an internal consistency check failed");
     else if (worst == SIM_E_STEPCAP) fail(c, SIM_E_STEPCAP, "sim_run: an instance hit the step cap");
     else if (worst == SIM_E_INFEASIBLE)
@@ -472,6 +497,35 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
         fail(c, SIM_E_INVAL, "sim_run: an instance violates 1 <= l <= o <= u, s >= 1, a >= 0 (rank >= 0 under A_r, "
                              "a < 2^30 under A_ell)");
     return worst;
+}
+
+int sim_set_tie_seeds(sim_ctx *c, const uint64_t *seeds) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    int rc = check_device(c);
+    if (rc) return rc;
+    if (!seeds) {
+        dfree(c->d_seed);
+        return SIM_OK;
+    }
+    cudaError_t e;
+    if (!c->d_seed && (e = dalloc(c->d_seed, size_t(c->n_inst) * sizeof(uint64_t))) != cudaSuccess)
+        return e == cudaErrorMemoryAllocation ? fail(c, SIM_E_NOMEM, "sim_set_tie_seeds: device allocation failed")
+                                              : cuda_fail(c, e, "cudaMalloc");
+    e = cudaMemcpy(c->d_seed, seeds, size_t(c->n_inst) * sizeof(uint64_t), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_set_tie_seeds: copy");
+    return SIM_OK;
+}
+
+int sim_get_work_counts(sim_ctx *c, int64_t *counts) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    if (!counts) return fail(c, SIM_E_INVAL, "sim_get_work_counts: NULL output");
+    if (!c->wc_valid || !c->d_wc)
+        return fail(c, SIM_E_STATE, "sim_get_work_counts: set SIM_OPT_COUNT_WORK=1 and call sim_run first");
+    cudaError_t e = cudaMemcpy(counts, c->d_wc, size_t(c->n_inst) * 4 * sizeof(int64_t), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_get_work_counts: copy");
+    return SIM_OK;
 }
 
 int sim_get_completions(sim_ctx *c, int64_t *completion_t) {
@@ -528,6 +582,8 @@ void sim_destroy(sim_ctx *c) {
     dfree(c->d_gws);
     dfree(c->d_main);
     dfree(c->d_cr);
+    dfree(c->d_seed);
+    dfree(c->d_wc);
     if (c->load_stream) cudaStreamDestroy(c->load_stream);
     if (c->h_off) cudaFreeHost(c->h_off);
     delete c;

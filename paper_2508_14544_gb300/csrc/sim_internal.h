@@ -48,6 +48,8 @@ struct StageParams {
     int64_t M;
     int32_t n_inst;
     int32_t n_max;             // largest instance (sizes the staging kernel's shared memory; 0: unknown)
+    int64_t max_total;         // capacity of rec / rec_a: an instance reaching past it is rejected (INVAL)
+    int32_t max_n;             // requests per instance above this are rejected (INVAL)
     int64_t step_cap;          // 0: default 64 * (n + sum o)
     const int64_t *off;        // n_inst + 1
     const int32_t *a, *s, *l, *u, *o;  // raw copies, n_total each
@@ -69,11 +71,15 @@ struct RunParams {
     DevResult *res;
     int64_t *completion;       // optional, n_total
     const int2 *lu;            // A_ell: (l, u) per request (staged), else null
+    const uint64_t *tie_seed;  // A_min: seed of the random eviction ties per instance, or null (0 for all)
+    int64_t *work_count;       // optional, 4 per instance: S2 adds, S3 compare-exchanges, S5 endpoint
+                               // evaluations of the per-step method, global bytes moved by the queue
     // workspace
     int32_t ca;                // active-set capacity per instance (multiple of 32)
     int32_t dcap;              // delta-queue capacity per instance (multiple of 32)
     int32_t use_smem;          // 1: active set + delta queue in shared memory; 0: global workspace
     int32_t debug;             // 1: check the simulation state's invariants every iteration (global kernel)
+    int32_t evict_index;       // 1: A_min eviction ties by request index instead of the random tie key
     unsigned char *gws;        // global workspace base (use_smem == 0)
     int64_t gws_stride;        // bytes per warp slot
     QEnt *mainbuf;             // ping-pong main-queue buffers, 2 * main_cap per warp slot

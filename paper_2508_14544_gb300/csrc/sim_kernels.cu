@@ -4,8 +4,10 @@
 // queue).  Each step follows the paper's algorithms:
 //   S1  arrivals with a_i <= t join the waiting set R_t (extension: the paper has a_i = 0);
 //   S3  A_min only (Algorithm milb): if the next step of the active set would exceed M, cancel
-//       jobs in ascending (estimate, index) order until it fits; each cancelled job's estimate
-//       becomes max(estimate, tokens generated) and it re-enters R_t in the same step;
+//       jobs in ascending estimate order, ties broken uniformly at random by a key drawn afresh
+//       at every step (SplitMix64 of the instance's seed and the counter t * 2^32 + index, then
+//       the index), until it fits; each cancelled job's estimate becomes max(estimate, tokens
+//       generated) and it re-enters R_t in the same step;
 //   S5  admit the largest prefix of R_t (sorted by (key, index)) for which eq. Constraint holds at
 //       every future step (Algorithms malb / milb / off);
 //   S6  process the batch: one token per member, the step's memory sum(s + tokens) (eq.
@@ -52,7 +54,7 @@ namespace {
 
 constexpr unsigned FULL = 0xffffffffu;
 enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2, P_AR = 3, P_AELL = 4 };
-enum { ST_OK = 0, ST_STEPCAP = -3, ST_STATE = -5 };
+enum { ST_OK = 0, ST_INVAL = -1, ST_STEPCAP = -3, ST_STATE = -5 };
 // Loops whose trip count is known only at run time carry `#pragma unroll 1`: their unrolled copies
 // added 15-20 % to the code of the simulation loop, which two warps on one scheduler share through
 // its instruction cache.
@@ -62,6 +64,24 @@ constexpr int kMc = 64;      // cached entries of the main queue (two per lane)
 constexpr int64_t kBig = int64_t(1) << 60;
 
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
+
+// Random tie key of request i at step t for A_min's cancellation order: the high 32 bits of
+// output number t * 2^32 + i + 1 of the SplitMix64 generator seeded with `seed` (Steele, Lea and
+// Flood, OOPSLA 2014, with the finalizer of Vigna's splitmix64.c): the state after k steps is
+// seed + k * 0x9E3779B97F4A7C15, mixed by two xor-shift-multiply rounds and a final xor-shift.
+// `base` = seed + t * 2^32 * 0x9E3779B97F4A7C15 (mod 2^64) is computed once per step.
+__device__ __forceinline__ uint64_t tie_base(uint64_t seed, int t) {
+    return seed + (uint64_t(uint32_t(t) * 0x7F4A7C15u) << 32);  // t * 2^32 * gamma mod 2^64
+}
+
+__device__ __forceinline__ unsigned tie_key(uint64_t base, int i) {
+    uint64_t z = base + uint64_t(uint32_t(i) + 1u) * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    z ^= z >> 31;
+    return unsigned(z >> 32);
+}
+
 
 __device__ __forceinline__ bool qless(const QEnt &a, const QEnt &b) {
     return a.key < b.key || (a.key == b.key && a.idx < b.idx);
@@ -294,6 +314,7 @@ struct Queue {
     int mbuf;        // -1: mq is read-only staged data; 0/1: ping-pong buffer in use
     int dn;          // delta size
     int mcb;         // main cache base: w.mc[i] = mq[mcb + i] for i < kMc; -1 invalid
+    int64_t gb;      // global-memory bytes the queue has moved (work counter)
 };
 
 __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.me && q.dn == 0; }
@@ -303,6 +324,7 @@ __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.m
 __device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
     if (q.mcb >= 0 && q.mh >= q.mcb && q.mh - q.mcb <= kMc - kWin) return;
     const int lane = lane_id();
+    q.gb += int64_t(min(kMc, q.me - q.mh)) * int64_t(sizeof(QEnt));
     const int i0 = q.mh + lane, i1 = q.mh + 32 + lane;
     QEnt a, b;
     if (i0 < q.me) a = q.mq[i0];
@@ -367,6 +389,7 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
     }
     __syncwarp();
     __threadfence_block();
+    q.gb += int64_t(2 * nx + dn) * int64_t(sizeof(QEnt));  // main read once, merged array written
     q.mq = out;
     q.mbuf = (q.mbuf == 0) ? 1 : 0;
     q.mh = 0;
@@ -440,6 +463,7 @@ __device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q) {
 __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
     const int lane = lane_id();
     if (len <= 0) return;
+    q.gb += int64_t(len) * int64_t(sizeof(QEnt));
     if (queue_empty(q)) {
         q.mq = run;
         q.mh = 0;
@@ -1097,7 +1121,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     r.total_latency = r.makespan = r.peak_memory = r.evictions = r.steps = r.request_steps = 0;
     r.status = info.status;
     r.pad = 0;
-    if (info.status != ST_OK || info.n == 0) {
+    if (info.status == ST_OK && int64_t(info.n) > P.main_cap) r.status = ST_INVAL;  // larger than the queue buffers
+    if (r.status != ST_OK || info.n == 0) {
         if (lane == 0) P.res[inst] = r;
         return;
     }
@@ -1107,12 +1132,6 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         return;
     }
     const int n = info.n;
-    // A_min cancellation order (estimate, index) as one 32-bit key when both fit: index bits kib
-    int kib = -1;
-    if (POL == P_AMIN) {
-        const int ib = 32 - __clz(max(n - 1, 1));
-        if (ib < 31 && (int64_t(info.lmax) + 1) <= (int64_t(1) << (32 - ib)) - 1) kib = ib;
-    }
     const QEnt *rec = P.rec + info.base;
     const int32_t *ra = P.rec_a + info.base;
     const int64_t M = P.M;
@@ -1124,6 +1143,13 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     q.mbuf = -1;
     q.dn = 0;
     q.mcb = -1;
+    q.gb = 0;
+    // work counters of the paper's per-step method (Theorem complexity), accumulated per step in
+    // closed form: S2 adds (the active set), S3 compare-exchanges of the overflow sort
+    // (A ceil(log2 A)^2), S5 endpoint evaluations of a binary-search admission
+    // ((A' + k) ceil(log2(Q + 1))); k_step / ev_step: admitted / removed at the current step
+    int64_t cS2 = 0, cS3 = 0, cS5 = 0;
+    int k_step = 0, ev_step = 0;
 
     int A = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
     if (lane == 0) {  // derived arrays of the empty active set (the workspace is reused)
@@ -1185,6 +1211,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 if (k < 32) break;
             }
             insert_run(w, q, rec + ap, ae - ap);
+            q.gb += int64_t(ae - ap) * 4;  // their arrival steps
             ap = ae;
             next_a = (ap < n) ? ra[ap] : INT_MAX;
             hvalid = false;
@@ -1197,60 +1224,53 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             t = next_a;  // idle: jump to the next arrival
             continue;
         }
-        // ---- S2/S3: A_min overflow of the next step -> cancel in ascending (estimate, index)
+        // ---- S2/S3: A_min overflow of the next step -> cancel in ascending (estimate, tie key, index)
         if (POL == P_AMIN) {
             wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
             if (need > wint<N>(M)) {
-                // one-chunk sets with packed keys: the keys stay in registers for all of the step's
-                // cancellations; a cancelled key becomes UINT_MAX
-                const bool reg = kib >= 0 && A <= kChunk;
-                unsigned key[4] = {UINT_MAX, UINT_MAX, UINT_MAX, UINT_MAX};
+                {
+                    const int lg = A > 1 ? 32 - __clz(A - 1) : 0;
+                    cS3 += int64_t(A) * lg * lg;
+                }
+                // Cancellation order (estimate, r, index), r the step's tie key (SplitMix64 of the seed
+                // and t * 2^32 + index; under the index rule r = index, the same order).  Estimate and
+                // r form one 64-bit key; two warp minima find the smallest, and an equal key held
+                // twice (a 32-bit collision of r, or the index rule) falls back to the index.
+                const uint64_t tb64 = tie_base(P.tie_seed ? P.tie_seed[inst] : 0ull, t);
+                const bool rnd = P.evict_index == 0;
+                // one-chunk sets: the lane's four keys stay in registers for all of the step's
+                // cancellations; a cancelled or missing entry holds the largest key
+                const bool reg = A <= kChunk;
+                uint64_t rk[4] = {~0ull, ~0ull, ~0ull, ~0ull};
+                int ri[4] = {0, 0, 0, 0};
                 if (reg) {
                     const int base = 4 * lane;
                     const int4 k4 = ld4(w.K, base), i4 = ld4(w.I, base);
                     const int kk[4] = {k4.x, k4.y, k4.z, k4.w}, ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        key[j] = (base + j < A) ? (unsigned(kk[j]) << kib) | unsigned(ii[j]) : UINT_MAX;
+                    for (int j = 0; j < 4; ++j) {
+                        ri[j] = ii[j];
+                        if (base + j < A)
+                            rk[j] = (uint64_t(uint32_t(kk[j])) << 32) | (rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]));
+                    }
                 }
                 #pragma unroll 1
                 while (need > wint<N>(M)) {
-                    int pos;
+                    // this lane's smallest key (and its index, smallest among equal keys)
+                    uint64_t bk = ~0ull;
+                    unsigned bi = UINT_MAX;
+                    int bp = -1;
                     if (reg) {
-                        // a min tree over this lane's four keys, then the position
-                        const unsigned best = min(min(key[0], key[1]), min(key[2], key[3]));
-                        const unsigned mk = __reduce_min_sync(FULL, best);
-                        const int j = key[0] == mk ? 0 : (key[1] == mk ? 1 : (key[2] == mk ? 2 : 3));
-                        const bool own = best == mk && mk != UINT_MAX;
-                        pos = int(__reduce_min_sync(FULL, own ? unsigned(4 * lane + j) : UINT_MAX));
+                        const uint64_t m01 = min(rk[0], rk[1]), m23 = min(rk[2], rk[3]);
+                        bk = min(m01, m23);
 #pragma unroll
-                        for (int m = 0; m < 4; ++m) key[m] = (own && m == j) ? UINT_MAX : key[m];
-                    } else if (kib >= 0) {
-                        // (estimate, index) packed into one 32-bit key: one reduction for the minimum
-                        unsigned best = UINT_MAX;
-                        int bp = -1;
-                        #pragma unroll 1
-                        for (int cb = 0; cb < A; cb += kChunk) {
-                            const int base = cb + 4 * lane;
-                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
-                            const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                const unsigned kj = (base + j < A && ff[j] >= 0)
-                                                        ? (unsigned(kk[j]) << kib) | unsigned(ii[j])
-                                                        : UINT_MAX;
-                                if (kj < best) {
-                                    best = kj;
-                                    bp = base + j;
-                                }
+                        for (int j = 0; j < 4; ++j) {
+                            if (rk[j] == bk && bk != ~0ull && unsigned(ri[j]) < bi) {
+                                bi = unsigned(ri[j]);
+                                bp = 4 * lane + j;
                             }
                         }
-                        const unsigned mk = __reduce_min_sync(FULL, best);
-                        pos = int(__reduce_min_sync(FULL, (bp >= 0 && best == mk) ? unsigned(bp) : UINT_MAX));
                     } else {
-                        unsigned bk = UINT_MAX, bi = UINT_MAX;
-                        int bp = -1;
                         #pragma unroll 1
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
@@ -1259,19 +1279,31 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                             const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
-                                if (base + j < A && ff[j] >= 0) {
-                                    const unsigned k = unsigned(kk[j]), i = unsigned(ii[j]);
-                                    if (k < bk || (k == bk && i < bi)) {
+                                if (base + j < A && ff[j] >= 0 && unsigned(kk[j]) <= unsigned(bk >> 32)) {
+                                    const uint64_t k = (uint64_t(uint32_t(kk[j])) << 32) |
+                                                       (rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]));
+                                    if (k < bk || (k == bk && unsigned(ii[j]) < bi)) {
                                         bk = k;
-                                        bi = i;
+                                        bi = unsigned(ii[j]);
                                         bp = base + j;
                                     }
                                 }
                             }
                         }
-                        const unsigned mk = __reduce_min_sync(FULL, bk);
-                        const unsigned mi = __reduce_min_sync(FULL, bk == mk ? bi : UINT_MAX);
-                        pos = int(__reduce_min_sync(FULL, (bp >= 0 && bk == mk && bi == mi) ? unsigned(bp) : UINT_MAX));
+                    }
+                    const unsigned mh = __reduce_min_sync(FULL, unsigned(bk >> 32));
+                    const unsigned ml = __reduce_min_sync(FULL, unsigned(bk >> 32) == mh ? unsigned(bk) : UINT_MAX);
+                    bool own = bp >= 0 && bk == ((uint64_t(mh) << 32) | ml);
+                    const unsigned ob = __ballot_sync(FULL, own);
+                    if (ob & (ob - 1)) {  // the smallest key in two lanes: the smaller index wins
+                        const unsigned mi = __reduce_min_sync(FULL, own ? bi : UINT_MAX);
+                        own = own && bi == mi;
+                    }
+                    const int pos = int(__reduce_min_sync(FULL, own ? unsigned(bp) : UINT_MAX));
+                    if (reg && own) {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            if (4 * lane + j == bp) rk[j] = ~0ull;
                     }
                     if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
@@ -1288,6 +1320,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     __syncwarp();
                     need -= wint<N>(b) + t;
                     ++nev;
+                    ++ev_step;
                     delta_insert(w, q, e);
                 }
                 if (status != ST_OK) break;
@@ -1319,6 +1352,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 delta_insert(w, q, e);
             }
             nev += c;
+            ev_step += c;
             tb_next = t;
             pend_compact = true;
             hvalid = false;
@@ -1371,6 +1405,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 status = ST_STATE;  // the head test and the window disagree: internal error
                 break;
             }
+            k_step += Kadm;
             const int cm = __popc(__ballot_sync(FULL, lane < Kadm && msrc == 0));
             q.mh += cm;
             q.dn -= Kadm - cm;
@@ -1406,6 +1441,12 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (mem > peak) peak = mem;
             rsteps += A;
             ++steps;
+            {
+                const int Qa = (q.me - q.mh) + q.dn;  // R_t after admission
+                cS2 += A - k_step + ev_step;
+                cS5 += int64_t(A) * (32 - __clz(Qa + k_step));
+                k_step = ev_step = 0;
+            }
             // the jobs with F = t complete (C = t + 1): the compaction at the top of the next
             // iteration removes them (F < the new time base) and counts them
             if (P.completion) {
@@ -1438,6 +1479,12 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (mem > peak) peak = mem;
             rsteps += int64_t(A) * c;
             steps += c;
+            {
+                const int Qa = (q.me - q.mh) + q.dn;
+                cS2 += int64_t(A) * c - k_step + ev_step;
+                cS5 += int64_t(A) * (32 - __clz(Qa + k_step)) + int64_t(A) * (c - 1) * (32 - __clz(Qa));
+                k_step = ev_step = 0;
+            }
             t += int(c);
         }
     }
@@ -1450,6 +1497,13 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         r.steps = steps;
         r.request_steps = rsteps;
         P.res[inst] = r;
+        if (P.work_count) {
+            int64_t *wc = P.work_count + 4 * int64_t(inst);
+            wc[0] = cS2;
+            wc[1] = cS3;
+            wc[2] = cS5;
+            wc[3] = q.gb;
+        }
     }
     __syncwarp();
 }

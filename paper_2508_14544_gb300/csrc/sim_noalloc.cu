@@ -129,6 +129,8 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     sp.M = M;
     sp.n_inst = n_instances;
     sp.n_max = int32_t(n_max);
+    sp.max_total = kNaMaxTotal;     // checked again on the device, against the offsets it reads
+    sp.max_n = int32_t(kNaMaxPerInstance);
     sp.step_cap = 0;
     sp.off = d_off;
     sp.a = arrival_t;
@@ -157,10 +159,13 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.res = reinterpret_cast<simgb::DevResult *>(results);
     p.completion = nullptr;
     p.lu = nullptr;
+    p.tie_seed = nullptr;  // seed 0 for every instance, as sim_run without sim_set_tie_seeds
+    p.work_count = nullptr;
     p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
     p.dcap = kNaDeltaCap;
     p.use_smem = 0;
     p.debug = 0;
+    p.evict_index = 0;
     p.gws = base + kOffWs;
     p.gws_stride = int64_t(ws_bytes_max());
     p.mainbuf = reinterpret_cast<simgb::QEnt *>(base + kOffMain);

@@ -106,8 +106,12 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
     extern __shared__ __align__(16) unsigned char stage_smem[];
     const int inst = blockIdx.x;
     const int64_t base = S.off[inst];
-    const int n = int(S.off[inst + 1] - base);
-    int64_t bad_inval = 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0;
+    const int64_t n64 = S.off[inst + 1] - base;
+    // offsets that reach outside the staged buffers (or above the per-instance limit) reject the
+    // instance before anything is written: it is staged as empty with status INVAL
+    const bool oob = base < 0 || n64 < 0 || n64 > S.max_n || base + n64 > S.max_total;
+    const int n = oob ? 0 : int(n64);
+    int64_t bad_inval = oob ? 1 : 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0;
     const bool in_smem = n <= np;
     uint64_t *sk = reinterpret_cast<uint64_t *>(stage_smem);
     int32_t *si = reinterpret_cast<int32_t *>(stage_smem + size_t(np) * 8);
@@ -160,7 +164,7 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
     else if (bad_inf) status = ST_INFEASIBLE;
     if (threadIdx.x == 0) {
         InstInfo in;
-        in.base = base;
+        in.base = oob ? 0 : base;
         in.n = n;
         in.status = status;
         in.sum_a = sum_a;

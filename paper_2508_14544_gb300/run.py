@@ -42,6 +42,7 @@ def main(argv=None) -> None:
     if args.warps_per_sm:
         opts["warps_per_sm"] = args.warps_per_sm
     with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
+        sim.set_tie_seeds(w.tie_seeds())
         for _ in range(args.repeat):
             sim.load(w.offsets, *dev, rank=rank)
             torch.cuda.synchronize()

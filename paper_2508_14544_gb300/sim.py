@@ -23,12 +23,19 @@ class Simulator:
     OPTIONS = {"step_cap": L.SIM_OPT_STEP_CAP, "record_completions": L.SIM_OPT_RECORD_COMPLETIONS,
                "warps_per_block": L.SIM_OPT_WARPS_PER_BLOCK, "smem_active_cap": L.SIM_OPT_SMEM_ACTIVE_CAP,
                "warps_per_sm": L.SIM_OPT_WARPS_PER_SM, "debug_checks": L.SIM_OPT_DEBUG_CHECKS,
-               "tune_residency": L.SIM_OPT_TUNE_RESIDENCY}
+               "tune_residency": L.SIM_OPT_TUNE_RESIDENCY, "evict_ties": L.SIM_OPT_EVICT_TIES,
+               "count_work": L.SIM_OPT_COUNT_WORK}
 
     def set_option(self, name: str, value: int) -> None:
         rc = L.sim_set_option(self.ctx, self.OPTIONS[name], int(value))
         if rc != L.SIM_OK:
             raise L.SimError(rc, L.sim_last_error(self.ctx))
+
+    def set_tie_seeds(self, seeds) -> None:
+        """Seeds of A_min's random cancellation ties, one per instance (None: all 0)."""
+        if seeds is not None:
+            assert len(seeds) == self.n_instances
+        self._check(L.sim_set_tie_seeds(self.ctx, seeds))
 
     def _check(self, rc: int, allow_instance_status: bool = False) -> int:
         if rc != L.SIM_OK and not (allow_instance_status and rc in (L.SIM_E_INVAL, L.SIM_E_INFEASIBLE,
@@ -54,14 +61,22 @@ class Simulator:
             self._check(L.sim_load_ranked_csr(self.ctx, offsets, *arrs, 1 if dev else 0))
 
     def load_workload(self, w) -> None:
-        """Load a seeded ``Workload``; under A_r its ranks() are the permutation."""
+        """Load a seeded ``Workload`` with its A_min tie seeds; under A_r its ranks() are the
+        permutation."""
         rank = w.ranks() if self.policy == L.SIM_AR else None
+        self.set_tie_seeds(w.tie_seeds())
         self.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o, rank=rank)
 
     def run(self, stream: int = 0) -> np.ndarray:
         out = np.zeros(self.n_instances, dtype=L.RESULT_DTYPE)
         self.last_rc = self._check(L.sim_run(self.ctx, out, stream), allow_instance_status=True)
         return out
+
+    def work_counts(self) -> np.ndarray:
+        """[n_instances, 4] int64 work counters of the last run (option count_work=1)."""
+        out = np.zeros(4 * self.n_instances, dtype=np.int64)
+        self._check(L.sim_get_work_counts(self.ctx, out))
+        return out.reshape(self.n_instances, 4)
 
     def completions(self, n_total: int) -> np.ndarray:
         out = np.zeros(max(n_total, 1), dtype=np.int64)

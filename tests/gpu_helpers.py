@@ -21,11 +21,13 @@ def gpu_run(policy, w, device_load=True, completions=False, rank=None, **opts):
         rank = w.ranks()
     with Simulator(policy, w.M, w.n_instances, record_completions=int(completions), **opts) as sim:
         if device_load:
+            sim.set_tie_seeds(w.tie_seeds())
             dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in
                    (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
             rk = None if rank is None else torch.from_numpy(np.ascontiguousarray(np.asarray(rank, np.int32))).cuda()
             sim.load(w.offsets, *dev, rank=rk)
         elif rank is not None:
+            sim.set_tie_seeds(w.tie_seeds())
             sim.load(w.offsets, w.arrival, w.prompt, w.lower, w.upper, w.true_o, rank=np.asarray(rank, np.int32))
         else:
             sim.load_workload(w)
@@ -34,9 +36,10 @@ def gpu_run(policy, w, device_load=True, completions=False, rank=None, **opts):
     return res, comp
 
 
-def oracle_run(policy, w, completions=False, step_cap=0):
+def oracle_run(policy, w, completions=False, step_cap=0, evict_ties="hash"):
     from oracle import plain
-    return plain.run_workload(policy, w, step_cap=step_cap, n_threads=n_threads(), completions=completions)
+    return plain.run_workload(policy, w, step_cap=step_cap, n_threads=n_threads(), completions=completions,
+                              evict_ties=evict_ties)
 
 
 def assert_same(got, ref, rows=None, tag=""):

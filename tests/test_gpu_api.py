@@ -228,11 +228,10 @@ def test_long_requests_narrow_and_wide_kernels_agree():
             assert np.array_equal(wide[f], ref[f]), (pol, f)
 
 
-def test_cancellation_order_without_packed_keys():
-    """A_min packs (estimate, index) into one 32-bit key when the instance's longest length and its
-    request count fit.  Here 4096 requests (12 index bits) and upper bounds of 1.2e6 (21 bits) do
-    not, so cancellations use the two-level (estimate, index) comparison; an instance of 1000
-    requests with short lengths next to it takes the packed path.  Both kernels equal the oracle."""
+def test_cancellation_order_with_long_bounds():
+    """A_min's cancellation order (estimate, random tie key, index) with upper bounds of 1.2e6 on a
+    4096-request instance, next to a 1000-request instance with short lengths: both kernels (the
+    shared-memory one and the checking global-memory one) equal the oracle."""
     from paper_2508_14544_gb300 import workloads as W
     rng = np.random.default_rng(33)
     parts = []

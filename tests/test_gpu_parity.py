@@ -19,9 +19,10 @@ def _cuda():
     g.build()
 
 
-def _gpu_sim(p, M, a, s, l, u, o, rank=None):
+def _gpu_sim(p, M, a, s, l, u, o, rank=None, tie_seed=0):
     from paper_2508_14544_gb300 import workloads as W
     w = W.concat_instances("pin", M, [dict(a=a, s=s, l=l, u=u, o=o)])
+    w.seed0 = int(tie_seed)  # the one instance's tie seed is seed0 + 0
     res, comp = gpu_run(p, w, completions=True, rank=rank)
     out = {k: int(res[0][k]) for k in FIELDS}
     out["completion"] = comp.tolist()
