@@ -71,6 +71,16 @@ Readings of the text that this oracle fixes (each is also listed in the design n
   when nothing is active or eligible, time jumps to the next arrival.  Makespan = max C_i.
 * Step cap.  A run that has processed ``step_cap`` batches without finishing stops with status
   STEPCAP.  Default cap: 64 * (n + sum_i o_i).
+* Batch time (Section 6: the experiments time each batch with a linear regression predictor).
+  The paper prints no coefficients, so the model is an input: a processed step t takes
+  f(B_t) = c0 + c1 |B_t| + c2 mem(t) + c3 prefill(t), where mem(t) is the step's memory (its KV
+  tokens) and prefill(t) the prompt tokens of the requests started at t; a step with nothing to
+  run takes c_idle.  A request's latency in time units is the time of the steps a_i .. C_i - 1.
+  Summed over the requests that latency is c0 X0 + c1 X1 + c2 X2 + c3 X3 with the integer sums
+  X_k = sum_i sum_{t in [a_i, C_i), processed} feature_k(t) (no step inside a request's interval
+  is idle), and the makespan in time units is c0 F0 + c1 F1 + c2 F2 + c3 F3 + c_idle F4 with the
+  feature totals F of steps 0 .. makespan - 1 (F4 the idle steps).  ``batch_time`` evaluates both
+  from the sums in that order, in IEEE double.
 """
 from __future__ import annotations
 
@@ -130,7 +140,22 @@ def validate(policy: int, M: int, a, s, l, u, o, rank=None) -> int:
 
 def _empty_result(status: int, n: int) -> dict:
     return dict(total_latency=0, makespan=0, peak_memory=0, evictions=0, steps=0,
-                request_steps=0, status=status, completion=[0] * n)
+                request_steps=0, status=status, completion=[0] * n, time_sums=[0] * 6)
+
+
+def batch_time(res: dict, coef: Sequence[float]) -> tuple[float, float]:
+    """(total latency, makespan) in time units under the linear batch-time model
+    coef = (c0, c1, c2, c3, c_idle), from a result's ``time_sums`` = [X0, X1, X2, X3, F2, F3]
+    (F0 = steps, F1 = request steps, F4 = makespan - steps), each a sum of products evaluated left
+    to right in IEEE double; NaN for an instance that did not finish."""
+    if res["status"] != OK:
+        return float("nan"), float("nan")
+    c0, c1, c2, c3, ci = (float(c) for c in coef)
+    x0, x1, x2, x3, f2, f3 = (float(v) for v in res["time_sums"])
+    tel = c0 * x0 + c1 * x1 + c2 * x2 + c3 * x3
+    span = (c0 * float(res["steps"]) + c1 * float(res["request_steps"]) + c2 * f2 + c3 * f3
+            + ci * float(res["makespan"] - res["steps"]))
+    return tel, span
 
 
 def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
@@ -173,6 +198,7 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
 
     tel = makespan = peak = evictions = steps = request_steps = 0
     status = OK
+    step_log = []  # (t, |B_t|, mem(t), prefill(t)) of every processed step
     t = min(a)
     n_done = 0
 
@@ -283,6 +309,7 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
             gen[i] += 1
         mem = sum(s[i] + gen[i] for i in batch)
         assert mem <= M, (t, mem, M)
+        step_log.append((t, len(batch), mem, sum(s[i] for i in admitted)))
         peak = max(peak, mem)
         request_steps += len(batch)
         steps += 1
@@ -307,8 +334,20 @@ def simulate(policy: int, M: int, a, s, l, u, o, step_cap: int | None = None,
                               evicted=list(evicted), finished=sorted(finished), mem=mem))
         t += 1
 
+    time_sums = [0] * 6
+    if status == OK:
+        for i in range(n):
+            for (tt, nb, mm, pf) in step_log:
+                if a[i] <= tt < completion[i]:
+                    time_sums[0] += 1
+                    time_sums[1] += nb
+                    time_sums[2] += mm
+                    time_sums[3] += pf
+        time_sums[4] = sum(mm for (_, _, mm, _) in step_log)
+        time_sums[5] = sum(pf for (_, _, _, pf) in step_log)
     return dict(total_latency=tel, makespan=makespan, peak_memory=peak, evictions=evictions,
-                steps=steps, request_steps=request_steps, status=status, completion=completion)
+                steps=steps, request_steps=request_steps, status=status, completion=completion,
+                time_sums=time_sums)
 
 
 def is_feasible_schedule(M: int, s: Sequence[int], o: Sequence[int], starts: Sequence[int]) -> bool:

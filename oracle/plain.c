@@ -24,9 +24,17 @@
  * grows linearly between two endpoints, so the maximum over t' >= t is reached at an endpoint;
  * at endpoint x the value is  sum_{e_j >= x} (s_j - p_j + 1 + x).
  *
+ * Batch time (Section 6, a linear batch-time predictor with caller-supplied coefficients): the
+ * optional time_sums output holds, per instance, X0..X3 = sum over requests of the number of
+ * processed steps, batch sizes, step memories and prefill (prompt tokens started) of the steps
+ * a_i .. C_i - 1, and F2, F3 = the totals of step memory and prefill over all processed steps.
+ * They are kept as prefix sums: an arrival at t subtracts the prefix up to t, a completion at C
+ * adds the prefix up to C.
+ *
  * Data structures are the textbook ones: a binary min-heap keyed by (key, index) for the waiting
  * set, an unsorted array for the active set, qsort for the endpoint sweep and the eviction order.
  */
+#include <math.h>
 #include <pthread.h>
 #include <stdint.h>
 #include <stdlib.h>
@@ -168,10 +176,12 @@ int64_t oracle_default_step_cap(int32_t n, const int32_t *o) {
  * rank (A_r only; may be NULL otherwise) is the permutation position of each request.
  * tie_seed seeds A_min's random eviction ties; evict_index != 0 breaks them by index instead.
  */
-int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
-                      const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
-                      uint64_t tie_seed, int evict_index, int64_t step_cap, oracle_result *res,
-                      int64_t *completion) {
+int oracle_run_full(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+                    const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                    uint64_t tie_seed, int evict_index, int64_t step_cap, oracle_result *res,
+                    int64_t *completion, int64_t *time_sums) {
+    if (time_sums)
+        for (int k = 0; k < 6; k++) time_sums[k] = 0;
     memset(res, 0, sizeof(*res));
     if (completion)
         for (int32_t i = 0; i < n; i++) completion[i] = 0;
@@ -214,6 +224,7 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
     qsort(arr, (size_t)n, sizeof(arr_t), cmp_arr);
 
     int64_t tel = 0, makespan = 0, peak = 0, evictions = 0, steps = 0, rsteps = 0;
+    int64_t memsum = 0, pfsum = 0, xs[4] = {0, 0, 0, 0}; /* batch-time prefix sums and X0..X3 */
     int32_t an = 0, n_done = 0, ap = 0;
     int64_t t = arr[0].a;
     int status = O_OK;
@@ -229,6 +240,10 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
         /* arrivals: requests with a_i <= t join the waiting set */
         while (ap < n && arr[ap].a <= t) {
             int32_t i = (int32_t)arr[ap].i;
+            xs[0] -= steps;
+            xs[1] -= rsteps;
+            xs[2] -= memsum;
+            xs[3] -= pfsum;
             heap_push(&q, ((uint64_t)QKEY(i) << 32) | (uint32_t)i);
             ap++;
         }
@@ -310,11 +325,12 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
         for (int32_t k = 0; k < nadm; k++) {
             start[nxt[k]] = t;
             act[an++] = nxt[k];
+            pfsum += s[nxt[k]];
         }
 
         /* process the batch: every member generates one token */
         int64_t mem = 0;
-        int32_t m = 0;
+        int32_t m = 0, ncomp = 0;
         for (int32_t k = 0; k < an; k++) {
             int32_t i = act[k];
             int64_t g = t - start[i] + 1;
@@ -325,6 +341,7 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
                 tel += C - a[i];
                 if (C > makespan) makespan = C;
                 n_done++;
+                ncomp++;
             } else {
                 act[m++] = i;
             }
@@ -333,6 +350,11 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
         an = m;
         if (mem > peak) peak = mem;
         steps++;
+        memsum += mem;
+        xs[0] += ncomp * steps; /* prefixes up to C = t + 1 */
+        xs[1] += ncomp * rsteps;
+        xs[2] += ncomp * memsum;
+        xs[3] += ncomp * pfsum;
         t++;
     }
 #undef QKEY
@@ -345,9 +367,22 @@ int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const 
     res->steps = steps;
     res->request_steps = rsteps;
     res->status = status;
+    if (time_sums && status == O_OK) {
+        for (int k = 0; k < 4; k++) time_sums[k] = xs[k];
+        time_sums[4] = memsum;
+        time_sums[5] = pfsum;
+    }
     free(start); free(otil); free(qkey); free(act); free(nxt); free(arr); free(ep); free(tmp);
     free(ev); free(q.v);
     return status;
+}
+
+int oracle_run_seeded(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
+                      const int32_t *l, const int32_t *u, const int32_t *o, const int32_t *rank,
+                      uint64_t tie_seed, int evict_index, int64_t step_cap, oracle_result *res,
+                      int64_t *completion) {
+    return oracle_run_full(policy, M, n, a, s, l, u, o, rank, tie_seed, evict_index, step_cap, res,
+                           completion, NULL);
 }
 
 int oracle_run_ex(int policy, int64_t M, int32_t n, const int32_t *a, const int32_t *s,
@@ -374,6 +409,7 @@ typedef struct {
     int64_t step_cap;
     oracle_result *res;
     int64_t *completion;
+    int64_t *time_sums;
     int32_t next;
     pthread_mutex_t mu;
 } batch_t;
@@ -386,21 +422,24 @@ static void *batch_worker(void *arg) {
         pthread_mutex_unlock(&b->mu);
         if (i >= b->n_inst) break;
         int64_t lo = b->off[i], hi = b->off[i + 1];
-        oracle_run_seeded(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
-                          b->u + lo, b->o + lo, b->rank ? b->rank + lo : NULL,
-                          b->tie_seed ? b->tie_seed[i] : 0, b->evict_index, b->step_cap, &b->res[i],
-                          b->completion ? b->completion + lo : NULL);
+        oracle_run_full(b->policy, b->M, (int32_t)(hi - lo), b->a + lo, b->s + lo, b->l + lo,
+                        b->u + lo, b->o + lo, b->rank ? b->rank + lo : NULL,
+                        b->tie_seed ? b->tie_seed[i] : 0, b->evict_index, b->step_cap, &b->res[i],
+                        b->completion ? b->completion + lo : NULL,
+                        b->time_sums ? b->time_sums + 6 * (int64_t)i : NULL);
     }
     return NULL;
 }
 
-/* Many instances (CSR offsets); tie_seed (optional, one per instance, else 0 for all). */
-int oracle_run_batch_seeded(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
-                            const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
-                            const int32_t *o, const int32_t *rank, const uint64_t *tie_seed,
-                            int evict_index, int64_t step_cap, oracle_result *res,
-                            int64_t *completion, int32_t n_threads) {
+/* Many instances (CSR offsets); tie_seed (optional, one per instance, else 0 for all);
+ * time_sums (optional, 6 per instance). */
+int oracle_run_batch_full(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                          const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                          const int32_t *o, const int32_t *rank, const uint64_t *tie_seed,
+                          int evict_index, int64_t step_cap, oracle_result *res,
+                          int64_t *completion, int64_t *time_sums, int32_t n_threads) {
     batch_t b;
+    b.time_sums = time_sums;
     b.policy = policy;
     b.M = M;
     b.n_inst = n_inst;
@@ -428,6 +467,15 @@ int oracle_run_batch_seeded(int policy, int64_t M, int32_t n_inst, const int64_t
     return worst;
 }
 
+int oracle_run_batch_seeded(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
+                            const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
+                            const int32_t *o, const int32_t *rank, const uint64_t *tie_seed,
+                            int evict_index, int64_t step_cap, oracle_result *res,
+                            int64_t *completion, int32_t n_threads) {
+    return oracle_run_batch_full(policy, M, n_inst, offsets, a, s, l, u, o, rank, tie_seed,
+                                 evict_index, step_cap, res, completion, NULL, n_threads);
+}
+
 int oracle_run_batch_ex(int policy, int64_t M, int32_t n_inst, const int64_t *offsets,
                         const int32_t *a, const int32_t *s, const int32_t *l, const int32_t *u,
                         const int32_t *o, const int32_t *rank, int64_t step_cap, oracle_result *res,
@@ -443,3 +491,25 @@ int oracle_run_batch(int policy, int64_t M, int32_t n_inst, const int64_t *offse
     return oracle_run_batch_ex(policy, M, n_inst, offsets, a, s, l, u, o, NULL, step_cap, res,
                                completion, n_threads);
 }
+
+/*
+ * Total latency and makespan in time units under the linear batch-time model
+ * coef = (c0, c1, c2, c3, c_idle) (Section 6): from time_sums = [X0, X1, X2, X3, F2, F3] and the
+ * result's steps (F0), request steps (F1) and makespan (F4 = makespan - steps),
+ *   out[0] = c0 X0 + c1 X1 + c2 X2 + c3 X3,
+ *   out[1] = c0 F0 + c1 F1 + c2 F2 + c3 F3 + c_idle F4,
+ * each evaluated left to right in IEEE double (built without contraction into fused multiply-adds);
+ * NaN for an instance that did not finish.
+ */
+void oracle_batch_time(const int64_t *time_sums, const oracle_result *res, const double *coef, double *out) {
+    if (res->status != O_OK) {
+        out[0] = out[1] = NAN;
+        return;
+    }
+    const double x0 = (double)time_sums[0], x1 = (double)time_sums[1], x2 = (double)time_sums[2];
+    const double x3 = (double)time_sums[3], f2 = (double)time_sums[4], f3 = (double)time_sums[5];
+    out[0] = coef[0] * x0 + coef[1] * x1 + coef[2] * x2 + coef[3] * x3;
+    out[1] = coef[0] * (double)res->steps + coef[1] * (double)res->request_steps + coef[2] * f2 +
+             coef[3] * f3 + coef[4] * (double)(res->makespan - res->steps);
+}
+
