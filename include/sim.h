@@ -115,9 +115,12 @@ enum {
                                        as Algorithm milb states (see sim_set_tie_seeds); 1: by the
                                        request index instead, a fixed order that always cancels the
                                        earliest-started of the tied jobs (for sensitivity studies). */
-    SIM_OPT_COUNT_WORK = 9          /* 0/1: record per instance the work that the paper's per-step
+    SIM_OPT_COUNT_WORK = 9,         /* 0/1: record per instance the work that the paper's per-step
                                        method does (sim_get_work_counts; default 0).  Results are
                                        identical; the counting costs a few instructions per event. */
+    SIM_OPT_BATCH_TIME = 10         /* 0/1: record per instance the integer sums that give total
+                                       latency and makespan in time units under a linear batch-time
+                                       model (sim_batch_time, sim_get_batch_time_sums; default 0). */
 };
 
 /*
@@ -216,6 +219,37 @@ int sim_set_tie_seeds(sim_ctx *ctx, const uint64_t *seeds);
  * (counting was off for the last sim_run) or SIM_E_CUDA.
  */
 int sim_get_work_counts(sim_ctx *ctx, int64_t *counts);
+
+/*
+ * sim_batch_time: total latency and makespan of every instance of the last sim_run in time units,
+ * under a linear batch-time model (Section 6 times each batch with a linear regression predictor;
+ * the paper prints no coefficients, so they are the caller's).  A processed step t with batch B_t
+ * takes
+ *     f(B_t) = c0 + c1 |B_t| + c2 mem(t) + c3 prefill(t),
+ * mem(t) = sum over B_t of (s_i + tokens), the step's KV tokens; prefill(t) = the prompt tokens of
+ * the requests started (or restarted) at t; a step with nothing to run takes c_idle.  Request i's
+ * latency in time units is the total time of steps a_i .. C_i - 1.
+ *   coef  HOST, 5 doubles: c0, c1, c2, c3, c_idle (finite).
+ *   out   HOST, 2 * n_instances doubles: [2i] = total latency in time units = c0 X0 + c1 X1 +
+ *         c2 X2 + c3 X3, [2i+1] = makespan in time units = c0 F0 + c1 F1 + c2 F2 + c3 F3 +
+ *         c_idle F4, each evaluated left to right in IEEE double without fused multiply-adds, with
+ *         the integer sums of sim_get_batch_time_sums (F0 = steps, F1 = request steps, F4 =
+ *         makespan - steps); NaN for an instance whose status is not SIM_OK.
+ * Requires SIM_OPT_BATCH_TIME = 1 before sim_run; coefficients can then change without
+ * re-simulating.  Synchronous on cuda_stream.  Returns SIM_OK, SIM_E_INVAL, SIM_E_STATE,
+ * SIM_E_NOMEM or SIM_E_CUDA.
+ */
+int sim_batch_time(sim_ctx *ctx, const double *coef, double *out, void *cuda_stream);
+
+/*
+ * sim_get_batch_time_sums: the integer sums behind sim_batch_time, six int64 per instance
+ * (HOST, 6 * n_instances): X0..X3 = sum over requests i of the number of processed steps, batch
+ * sizes |B_t|, step memories mem(t) and prefill tokens prefill(t) of the steps a_i .. C_i - 1 (no
+ * step inside a request's interval is idle); F2, F3 = the totals of mem(t) and prefill(t) over
+ * all processed steps.  Zeros for an instance whose status is not SIM_OK.  X2 stays exact while
+ * M * total latency < 2^63.  Returns SIM_OK, SIM_E_INVAL, SIM_E_STATE or SIM_E_CUDA.
+ */
+int sim_get_batch_time_sums(sim_ctx *ctx, int64_t *sums);
 
 /*
  * sim_get_completions: copy every request's completion step C_i of the last sim_run into

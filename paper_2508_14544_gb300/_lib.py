@@ -21,6 +21,7 @@ SIM_OPT_DEBUG_CHECKS = 6
 SIM_OPT_TUNE_RESIDENCY = 7
 SIM_OPT_EVICT_TIES = 8
 SIM_OPT_COUNT_WORK = 9
+SIM_OPT_BATCH_TIME = 10
 
 STATUS_NAMES = {0: "SIM_OK", -1: "SIM_E_INVAL", -2: "SIM_E_INFEASIBLE", -3: "SIM_E_STEPCAP", -4: "SIM_E_CUDA",
                 -5: "SIM_E_STATE", -6: "SIM_E_NOMEM"}
@@ -39,7 +40,8 @@ RESULT_DTYPE = np.dtype([
 assert RESULT_DTYPE.itemsize == ctypes.sizeof(sim_result) == 56
 
 EXPORTS = ("sim_create", "sim_load", "sim_load_csr", "sim_load_ranked_csr", "sim_run", "sim_get_completions", "sim_competitive_ratio",
-           "sim_set_option", "sim_set_tie_seeds", "sim_get_work_counts", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc",
+           "sim_set_option", "sim_set_tie_seeds", "sim_get_work_counts", "sim_batch_time",
+           "sim_get_batch_time_sums", "sim_last_error", "sim_destroy", "sim_kernel_launches", "sim_run_noalloc",
            "sim_cr_amin_lemma", "sim_cr_amin_rho", "sim_measure_peaks")
 
 _lib = None
@@ -86,6 +88,10 @@ def lib() -> ctypes.CDLL:
     L.sim_set_tie_seeds.restype = ctypes.c_int
     L.sim_get_work_counts.argtypes = [vp, vp]
     L.sim_get_work_counts.restype = ctypes.c_int
+    L.sim_batch_time.argtypes = [vp, vp, vp, vp]
+    L.sim_batch_time.restype = ctypes.c_int
+    L.sim_get_batch_time_sums.argtypes = [vp, vp]
+    L.sim_get_batch_time_sums.restype = ctypes.c_int
     L.sim_last_error.argtypes = [vp]
     L.sim_last_error.restype = ctypes.c_char_p
     L.sim_destroy.argtypes = [vp]
@@ -165,6 +171,17 @@ def sim_run(ctx, out: np.ndarray, stream: int = 0) -> int:
 def sim_get_work_counts(ctx, out: np.ndarray) -> int:
     assert out.dtype == np.int64 and out.flags.c_contiguous
     return lib().sim_get_work_counts(ctx, out.ctypes.data)
+
+
+def sim_batch_time(ctx, coef, out: np.ndarray, stream: int = 0) -> int:
+    cf = np.ascontiguousarray(np.asarray(coef, dtype=np.float64))
+    assert cf.shape == (5,) and out.dtype == np.float64 and out.flags.c_contiguous
+    return lib().sim_batch_time(ctx, cf.ctypes.data, out.ctypes.data, ctypes.c_void_p(stream or None))
+
+
+def sim_get_batch_time_sums(ctx, out: np.ndarray) -> int:
+    assert out.dtype == np.int64 and out.flags.c_contiguous
+    return lib().sim_get_batch_time_sums(ctx, out.ctypes.data)
 
 
 def sim_get_completions(ctx, out: np.ndarray) -> int:

@@ -33,6 +33,7 @@ struct sim_ctx {
     int tune_residency = 0;
     int evict_index = 0;
     int count_work = 0;
+    int batch_time = 0;
     // residency chosen by SIM_OPT_TUNE_RESIDENCY for the load shape tuned_shape (n_inst, n_total,
     // n_max): warps per SM, or 0 for the default; tuned_shape[0] < 0 when not tuned
     int tuned_wps = 0;
@@ -66,6 +67,9 @@ struct sim_ctx {
     uint64_t *d_seed = nullptr;          // A_min tie seeds (n_inst), null until sim_set_tie_seeds
     int64_t *d_wc = nullptr;             // work counters, 4 per instance (SIM_OPT_COUNT_WORK)
     bool wc_valid = false;
+    int64_t *d_bt = nullptr;             // batch-time sums, 6 per instance (SIM_OPT_BATCH_TIME)
+    double *d_btout = nullptr;           // 2 per instance
+    bool bt_valid = false;
     cudaStream_t load_stream = nullptr;  // non-blocking stream of sim_load (independent of other threads' work)
     int64_t *h_off = nullptr;            // pinned copy of the offsets (n_inst + 1) for their upload
     int64_t launches = 0;
@@ -180,6 +184,9 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
             return SIM_OK;
         case SIM_OPT_COUNT_WORK:
             c->count_work = value ? 1 : 0;
+            return SIM_OK;
+        case SIM_OPT_BATCH_TIME:
+            c->batch_time = value ? 1 : 0;
             return SIM_OK;
         case SIM_OPT_SMEM_ACTIVE_CAP:
             if (value < 128 || value > 4096 || value % 128)
@@ -377,6 +384,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.lu = c->d_lu;
     p.tie_seed = c->d_seed;
     p.work_count = c->count_work ? c->d_wc : nullptr;
+    p.batch_time = c->batch_time ? c->d_bt : nullptr;
     p.ca = ca;
     p.dcap = dcap;
     p.use_smem = smem ? 1 : 0;
@@ -411,6 +419,10 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
             return cuda_fail(c, e, "cudaMemsetAsync");
     }
     c->wc_valid = false;
+    c->bt_valid = false;
+    if (c->batch_time && !c->d_bt &&
+        (e = dalloc(c->d_bt, size_t(c->n_inst) * 6 * sizeof(int64_t))) != cudaSuccess)
+        return fail(c, SIM_E_NOMEM, "sim_run: batch-time buffer");
     if (c->count_work) {
         if (!c->d_wc && (e = dalloc(c->d_wc, size_t(c->n_inst) * 4 * sizeof(int64_t))) != cudaSuccess)
             return fail(c, SIM_E_NOMEM, "sim_run: work-counter buffer");
@@ -489,6 +501,7 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
     c->ran = true;
     c->comp_valid = c->record_completions != 0;
     c->wc_valid = c->count_work != 0;
+    c->bt_valid = c->batch_time != 0;
     if (worst == SIM_E_STATE) fail(c, SIM_E_STATE, "sim_run: an internal consistency check failed");
     else if (worst == SIM_E_STEPCAP) fail(c, SIM_E_STEPCAP, "sim_run: an instance hit the step cap");
     else if (worst == SIM_E_INFEASIBLE)
@@ -525,6 +538,42 @@ int sim_get_work_counts(sim_ctx *c, int64_t *counts) {
         return fail(c, SIM_E_STATE, "sim_get_work_counts: set SIM_OPT_COUNT_WORK=1 and call sim_run first");
     cudaError_t e = cudaMemcpy(counts, c->d_wc, size_t(c->n_inst) * 4 * sizeof(int64_t), cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_get_work_counts: copy");
+    return SIM_OK;
+}
+
+int sim_get_batch_time_sums(sim_ctx *c, int64_t *sums) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    if (!sums) return fail(c, SIM_E_INVAL, "sim_get_batch_time_sums: NULL output");
+    if (!c->bt_valid || !c->d_bt)
+        return fail(c, SIM_E_STATE, "sim_get_batch_time_sums: set SIM_OPT_BATCH_TIME=1 and call sim_run first");
+    cudaError_t e = cudaMemcpy(sums, c->d_bt, size_t(c->n_inst) * 6 * sizeof(int64_t), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_get_batch_time_sums: copy");
+    return SIM_OK;
+}
+
+int sim_batch_time(sim_ctx *c, const double *coef, double *out, void *stream) {
+    if (!c) return SIM_E_INVAL;
+    c->err.clear();
+    if (!coef || !out) return fail(c, SIM_E_INVAL, "sim_batch_time: NULL coefficients or output");
+    for (int k = 0; k < 5; ++k)
+        if (!(coef[k] == coef[k]) || coef[k] - coef[k] != 0.0)
+            return fail(c, SIM_E_INVAL, "sim_batch_time: coefficient %d is not finite", k);
+    if (!c->bt_valid || !c->d_bt)
+        return fail(c, SIM_E_STATE, "sim_batch_time: set SIM_OPT_BATCH_TIME=1 and call sim_run first");
+    int rc = check_device(c);
+    if (rc) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if (!c->d_btout && (e = dalloc(c->d_btout, size_t(c->n_inst) * 2 * sizeof(double))) != cudaSuccess)
+        return fail(c, SIM_E_NOMEM, "sim_batch_time: buffer");
+    e = simgb::launch_batch_time(c->d_bt, c->d_res, coef, c->d_btout, c->n_inst, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_batch_time: launch");
+    ++c->launches;
+    e = cudaMemcpyAsync(out, c->d_btout, size_t(c->n_inst) * 2 * sizeof(double), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_batch_time: copy");
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sim_batch_time: sync");
     return SIM_OK;
 }
 
@@ -584,6 +633,8 @@ void sim_destroy(sim_ctx *c) {
     dfree(c->d_cr);
     dfree(c->d_seed);
     dfree(c->d_wc);
+    dfree(c->d_bt);
+    dfree(c->d_btout);
     if (c->load_stream) cudaStreamDestroy(c->load_stream);
     if (c->h_off) cudaFreeHost(c->h_off);
     delete c;

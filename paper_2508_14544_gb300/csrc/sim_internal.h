@@ -74,6 +74,7 @@ struct RunParams {
     const uint64_t *tie_seed;  // A_min: seed of the random eviction ties per instance, or null (0 for all)
     int64_t *work_count;       // optional, 4 per instance: S2 adds, S3 compare-exchanges, S5 endpoint
                                // evaluations of the per-step method, global bytes moved by the queue
+    int64_t *batch_time;       // optional, 6 per instance: the batch-time sums X0..X3, F2, F3
     // workspace
     int32_t ca;                // active-set capacity per instance (multiple of 32)
     int32_t dcap;              // delta-queue capacity per instance (multiple of 32)
@@ -92,6 +93,8 @@ cudaError_t launch_stage(const StageParams &p, cudaStream_t st);
 cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
                        cudaStream_t st);
 cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
+cudaError_t launch_batch_time(const int64_t *sums, const DevResult *res, const double *coef, double *out, int32_t n,
+                              cudaStream_t st);
 cudaError_t set_run_smem_limit(int policy, size_t bytes);
 cudaError_t launch_lemma(int32_t n_hist, int32_t len, int32_t l, double s, const double *x, double *out,
                          cudaStream_t st);

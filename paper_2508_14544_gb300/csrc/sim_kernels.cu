@@ -1,4 +1,4 @@
-// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared>.
+// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared, instrumented>.
 //
 // One warp simulates one instance at a time (persistent warps pull instance ids from a work
 // queue).  Each step follows the paper's algorithms:
@@ -1108,8 +1108,10 @@ __device__ bool state_ok(const Ws &w, const Queue &q, int A, int tb, int SB0, in
 
 // ---------------------------------------------------------------------------------------------
 // One instance, simulated by one warp.  All lanes hold identical copies of the scalar state.
+// INS: the instrumented copy, which also keeps the work counters of the per-step method and the
+// batch-time sums; the plain copy has neither.
 // ---------------------------------------------------------------------------------------------
-template <int POL, bool N>
+template <int POL, bool N, bool INS>
 __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, int inst) {
     const int lane = lane_id();
     const InstInfo info = P.info[inst];
@@ -1134,6 +1136,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     const int n = info.n;
     const QEnt *rec = P.rec + info.base;
     const int32_t *ra = P.rec_a + info.base;
+    const uint64_t tie_seed = (POL == P_AMIN && P.tie_seed) ? P.tie_seed[inst] : 0ull;
+    // bits of the longest length (every A_min estimate is below 2^kbits), for the packed
+    // cancellation keys
+    const int kbits = 32 - __clz(max(info.lmax, 1));
     const int64_t M = P.M;
     const int64_t cap = info.cap;
 
@@ -1151,6 +1157,13 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     int64_t cS2 = 0, cS3 = 0, cS5 = 0;
     int k_step = 0, ev_step = 0;
 
+    // Batch time (Section 6's linear batch-time model, coefficients given later): bx0..bx3 =
+    // X0..X3, the sums over requests of the processed steps, batch sizes, step memories and
+    // prefill tokens of the steps a_i .. C_i - 1 (an arrival at t subtracts the prefixes up to t,
+    // a completion at C adds those up to C); bmem, bpf the prefixes of step memory and prefill
+    // (steps and request steps have their own counters).
+    const bool bt = INS && P.batch_time != nullptr;
+    int64_t bx0 = 0, bx1 = 0, bx2 = 0, bx3 = 0, bmem = 0, bpf = 0;
     int A = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
     if (lane == 0) {  // derived arrays of the empty active set (the workspace is reused)
         w.SB[0] = 0;
@@ -1187,6 +1200,12 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (done_step) {  // the jobs completed at step tb - 1 (C = tb) have left the set
                 const int c = A0 - A;
                 sumC += int64_t(c) * tb;
+                if (bt) {
+                    bx0 += int64_t(c) * steps;
+                    bx1 += int64_t(c) * rsteps;
+                    bx2 += int64_t(c) * bmem;
+                    bx3 += int64_t(c) * bpf;
+                }
                 ndone += c;
                 done_step = false;
                 if (ndone >= n) break;
@@ -1211,7 +1230,14 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 if (k < 32) break;
             }
             insert_run(w, q, rec + ap, ae - ap);
-            q.gb += int64_t(ae - ap) * 4;  // their arrival steps
+            if (INS) q.gb += int64_t(ae - ap) * 4;  // their arrival steps
+            if (bt) {
+                const int64_t m = ae - ap;
+                bx0 -= m * steps;
+                bx1 -= m * rsteps;
+                bx2 -= m * bmem;
+                bx3 -= m * bpf;
+            }
             ap = ae;
             next_a = (ap < n) ? ra[ap] : INT_MAX;
             hvalid = false;
@@ -1228,21 +1254,23 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         if (POL == P_AMIN) {
             wint<N> need = wint<N>(SB0) + wint<N>(A) * (t - tb);
             if (need > wint<N>(M)) {
-                {
+                if (INS) {
                     const int lg = A > 1 ? 32 - __clz(A - 1) : 0;
                     cS3 += int64_t(A) * lg * lg;
                 }
                 // Cancellation order (estimate, r, index), r the step's tie key (SplitMix64 of the seed
-                // and t * 2^32 + index; under the index rule r = index, the same order).  Estimate and
-                // r form one 64-bit key; two warp minima find the smallest, and an equal key held
-                // twice (a 32-bit collision of r, or the index rule) falls back to the index.
-                const uint64_t tb64 = tie_base(P.tie_seed ? P.tie_seed[inst] : 0ull, t);
+                // and t * 2^32 + index; under the index rule r = index, the same order).
+                const uint64_t tb64 = tie_base(tie_seed, t);
                 const bool rnd = P.evict_index == 0;
-                // one-chunk sets: the lane's four keys stay in registers for all of the step's
-                // cancellations; a cancelled or missing entry holds the largest key
+                // One-chunk sets: the lane's four entries are keyed once per step, in registers, by
+                // pk = estimate << (32 - kb) | r >> kb (estimate < 2^kb), whose order is that of
+                // (estimate, high bits of r); a round takes one warp minimum of pk, and only equal pk
+                // (the same estimate and the same high bits of r) look at all of r, then the index.
+                // A cancelled or missing entry holds pk = UINT_MAX and is never a candidate.
                 const bool reg = A <= kChunk;
-                uint64_t rk[4] = {~0ull, ~0ull, ~0ull, ~0ull};
+                unsigned pk[4] = {UINT_MAX, UINT_MAX, UINT_MAX, UINT_MAX}, rr[4] = {0u, 0u, 0u, 0u};
                 int ri[4] = {0, 0, 0, 0};
+                unsigned live = 0;  // bit j: entry j of the lane is a live job
                 if (reg) {
                     const int base = 4 * lane;
                     const int4 k4 = ld4(w.K, base), i4 = ld4(w.I, base);
@@ -1250,60 +1278,108 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         ri[j] = ii[j];
-                        if (base + j < A)
-                            rk[j] = (uint64_t(uint32_t(kk[j])) << 32) | (rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]));
+                        if (base + j < A) {
+                            live |= 1u << j;
+                            rr[j] = rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]);
+                            pk[j] = (unsigned(kk[j]) << (32 - kbits)) | (kbits == 32 ? 0u : rr[j] >> kbits);
+                        }
                     }
                 }
                 #pragma unroll 1
                 while (need > wint<N>(M)) {
-                    // this lane's smallest key (and its index, smallest among equal keys)
-                    uint64_t bk = ~0ull;
-                    unsigned bi = UINT_MAX;
-                    int bp = -1;
+                    int pos = -1;
                     if (reg) {
-                        const uint64_t m01 = min(rk[0], rk[1]), m23 = min(rk[2], rk[3]);
-                        bk = min(m01, m23);
+                        const unsigned mk = __reduce_min_sync(FULL, min(min(pk[0], pk[1]), min(pk[2], pk[3])));
+                        unsigned cand = 0;  // bit j: entry j holds the smallest packed key
+                        int tot = 0;
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
-                            if (rk[j] == bk && bk != ~0ull && unsigned(ri[j]) < bi) {
-                                bi = unsigned(ri[j]);
-                                bp = 4 * lane + j;
+                            const bool c = ((live >> j) & 1u) && pk[j] == mk;
+                            cand |= c ? (1u << j) : 0u;
+                            const unsigned b = __ballot_sync(FULL, c);
+                            tot += __popc(b);
+                            if (b) pos = 4 * (__ffs(b) - 1) + j;
+                        }
+                        if (tot > 1) {  // equal packed keys: all of r, then the index
+                            unsigned lr = UINT_MAX;
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                if ((cand >> j) & 1u) lr = min(lr, rr[j]);
+                            const unsigned mr = __reduce_min_sync(FULL, lr);
+                            unsigned li = UINT_MAX;
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                if (rr[j] != mr) cand &= ~(1u << j);
+                                if ((cand >> j) & 1u) li = min(li, unsigned(ri[j]));
+                            }
+                            const unsigned mi = __reduce_min_sync(FULL, li);
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                const unsigned b = __ballot_sync(FULL, ((cand >> j) & 1u) && unsigned(ri[j]) == mi);
+                                if (b) pos = 4 * (__ffs(b) - 1) + j;
                             }
                         }
+                        if (pos >= 0 && (pos >> 2) == lane) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                if ((pos & 3) == j) pk[j] = UINT_MAX;
+                            live &= ~(1u << (pos & 3));
+                        }
                     } else {
+                        // wider sets: one pass for the smallest estimate, how many live jobs share it
+                        // and (if one) where; a second pass draws the tied jobs' keys otherwise
+                        unsigned bk = UINT_MAX;
+                        int bc = 0, bp = -1;
                         #pragma unroll 1
                         for (int cb = 0; cb < A; cb += kChunk) {
                             const int base = cb + 4 * lane;
-                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                            const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base);
                             const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-                            const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
-                                if (base + j < A && ff[j] >= 0 && unsigned(kk[j]) <= unsigned(bk >> 32)) {
-                                    const uint64_t k = (uint64_t(uint32_t(kk[j])) << 32) |
-                                                       (rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]));
-                                    if (k < bk || (k == bk && unsigned(ii[j]) < bi)) {
+                                if (base + j < A && ff[j] >= 0) {
+                                    const unsigned k = unsigned(kk[j]);
+                                    if (k < bk) {
                                         bk = k;
-                                        bi = unsigned(ii[j]);
+                                        bc = 1;
                                         bp = base + j;
+                                    } else if (k == bk) {
+                                        ++bc;
                                     }
                                 }
                             }
                         }
-                    }
-                    const unsigned mh = __reduce_min_sync(FULL, unsigned(bk >> 32));
-                    const unsigned ml = __reduce_min_sync(FULL, unsigned(bk >> 32) == mh ? unsigned(bk) : UINT_MAX);
-                    bool own = bp >= 0 && bk == ((uint64_t(mh) << 32) | ml);
-                    const unsigned ob = __ballot_sync(FULL, own);
-                    if (ob & (ob - 1)) {  // the smallest key in two lanes: the smaller index wins
-                        const unsigned mi = __reduce_min_sync(FULL, own ? bi : UINT_MAX);
-                        own = own && bi == mi;
-                    }
-                    const int pos = int(__reduce_min_sync(FULL, own ? unsigned(bp) : UINT_MAX));
-                    if (reg && own) {
+                        const unsigned mk = __reduce_min_sync(FULL, bk);
+                        const int tot = int(__reduce_add_sync(FULL, bk == mk ? unsigned(bc) : 0u));
+                        if (mk != UINT_MAX && tot == 1) {
+                            const unsigned b = __ballot_sync(FULL, bk == mk && bc > 0);
+                            pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
+                        } else if (mk != UINT_MAX) {
+                            unsigned br = UINT_MAX, bi = UINT_MAX;
+                            bp = -1;
+                            #pragma unroll 1
+                            for (int cb = 0; cb < A; cb += kChunk) {
+                                const int base = cb + 4 * lane;
+                                const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
+                                const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                                const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            if (4 * lane + j == bp) rk[j] = ~0ull;
+                                for (int j = 0; j < 4; ++j) {
+                                    if (base + j < A && ff[j] >= 0 && unsigned(kk[j]) == mk) {
+                                        const unsigned r = rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]);
+                                        if (r < br || (r == br && unsigned(ii[j]) < bi)) {
+                                            br = r;
+                                            bi = unsigned(ii[j]);
+                                            bp = base + j;
+                                        }
+                                    }
+                                }
+                            }
+                            const unsigned mr = __reduce_min_sync(FULL, br);
+                            const unsigned mi = __reduce_min_sync(FULL, br == mr ? bi : UINT_MAX);
+                            const unsigned b = __ballot_sync(FULL, bp >= 0 && br == mr && bi == mi);
+                            pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
+                        }
                     }
                     if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
@@ -1320,7 +1396,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     __syncwarp();
                     need -= wint<N>(b) + t;
                     ++nev;
-                    ++ev_step;
+                    if (INS) ++ev_step;
                     delta_insert(w, q, e);
                 }
                 if (status != ST_OK) break;
@@ -1352,7 +1428,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 delta_insert(w, q, e);
             }
             nev += c;
-            ev_step += c;
+            if (INS) ev_step += c;
             tb_next = t;
             pend_compact = true;
             hvalid = false;
@@ -1405,7 +1481,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 status = ST_STATE;  // the head test and the window disagree: internal error
                 break;
             }
-            k_step += Kadm;
+            if (INS) k_step += Kadm;
+            if (bt)  // prefill: the prompts of the admitted requests
+                bpf += int64_t(__reduce_add_sync(FULL, lane < Kadm ? unsigned(mine.s) : 0u));
             const int cm = __popc(__ballot_sync(FULL, lane < Kadm && msrc == 0));
             q.mh += cm;
             q.dn -= Kadm - cm;
@@ -1441,7 +1519,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (mem > peak) peak = mem;
             rsteps += A;
             ++steps;
-            {
+            if (bt) bmem += int64_t(mem);
+            if (INS) {
                 const int Qa = (q.me - q.mh) + q.dn;  // R_t after admission
                 cS2 += A - k_step + ev_step;
                 cS5 += int64_t(A) * (32 - __clz(Qa + k_step));
@@ -1479,7 +1558,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (mem > peak) peak = mem;
             rsteps += int64_t(A) * c;
             steps += c;
-            {
+            if (bt)  // steps t .. t+c-1 have memory SB0 + A (x - tb)
+                bmem += c * int64_t(SB0) + int64_t(A) * (c * (int64_t(t) - tb) + c * (c - 1) / 2);
+            if (INS) {
                 const int Qa = (q.me - q.mh) + q.dn;
                 cS2 += int64_t(A) * c - k_step + ev_step;
                 cS5 += int64_t(A) * (32 - __clz(Qa + k_step)) + int64_t(A) * (c - 1) * (32 - __clz(Qa));
@@ -1497,7 +1578,17 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         r.steps = steps;
         r.request_steps = rsteps;
         P.res[inst] = r;
-        if (P.work_count) {
+        if (bt) {
+            int64_t *o = P.batch_time + 6 * int64_t(inst);
+            const bool ok = status == ST_OK;
+            o[0] = ok ? bx0 : 0;
+            o[1] = ok ? bx1 : 0;
+            o[2] = ok ? bx2 : 0;
+            o[3] = ok ? bx3 : 0;
+            o[4] = ok ? bmem : 0;
+            o[5] = ok ? bpf : 0;
+        }
+        if (INS && P.work_count) {
             int64_t *wc = P.work_count + 4 * int64_t(inst);
             wc[0] = cS2;
             wc[1] = cS3;
@@ -1508,7 +1599,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     __syncwarp();
 }
 
-template <int POL, bool SMEM>
+template <int POL, bool SMEM, bool INS>
 __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
@@ -1526,13 +1617,27 @@ __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
         k = __shfl_sync(FULL, k, 0);
         if (k >= P.n_work) break;
         const int inst = P.work ? P.work[k] : k;
-        sim_instance<POL, SMEM>(P, w, inst);
+        sim_instance<POL, SMEM, INS>(P, w, inst);
     }
 }
 
 template <int POL>
-const void *run_fn(bool smem) {
-    return smem ? (const void *)k_run<POL, true> : (const void *)k_run<POL, false>;
+const void *run_fn(bool smem, bool ins) {
+    if (ins) return smem ? (const void *)k_run<POL, true, true> : (const void *)k_run<POL, false, true>;
+    return smem ? (const void *)k_run<POL, true, false> : (const void *)k_run<POL, false, false>;
+}
+
+template <int POL>
+void launch_pol(const RunParams &p, dim3 grid, dim3 block, size_t smem_bytes, cudaStream_t st) {
+    const bool sm = p.use_smem != 0;
+    const bool ins = p.work_count != nullptr || p.batch_time != nullptr;
+    if (ins) {
+        if (sm) k_run<POL, true, true><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, true><<<grid, block, smem_bytes, st>>>(p);
+    } else {
+        if (sm) k_run<POL, true, false><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, false><<<grid, block, smem_bytes, st>>>(p);
+    }
 }
 
 }  // namespace
@@ -1540,39 +1645,27 @@ const void *run_fn(bool smem) {
 size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
-    const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true)
-                     : policy == P_AMIN ? run_fn<P_AMIN>(true)
-                     : policy == P_HSF  ? run_fn<P_HSF>(true)
-                     : policy == P_AR   ? run_fn<P_AR>(true)
-                                        : run_fn<P_AELL>(true);
-    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
+    for (int ins = 0; ins < 2; ++ins) {
+        const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true, ins)
+                         : policy == P_AMIN ? run_fn<P_AMIN>(true, ins)
+                         : policy == P_HSF  ? run_fn<P_HSF>(true, ins)
+                         : policy == P_AR   ? run_fn<P_AR>(true, ins)
+                                            : run_fn<P_AELL>(true, ins);
+        const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
                        cudaStream_t st) {
     const dim3 grid(blocks), block(32 * warps_per_block);
-    const bool sm = p.use_smem != 0;
     switch (policy) {
-        case P_AMAX:
-            if (sm) k_run<P_AMAX, true><<<grid, block, smem_bytes, st>>>(p);
-            else k_run<P_AMAX, false><<<grid, block, smem_bytes, st>>>(p);
-            break;
-        case P_AMIN:
-            if (sm) k_run<P_AMIN, true><<<grid, block, smem_bytes, st>>>(p);
-            else k_run<P_AMIN, false><<<grid, block, smem_bytes, st>>>(p);
-            break;
-        case P_HSF:
-            if (sm) k_run<P_HSF, true><<<grid, block, smem_bytes, st>>>(p);
-            else k_run<P_HSF, false><<<grid, block, smem_bytes, st>>>(p);
-            break;
-        case P_AR:
-            if (sm) k_run<P_AR, true><<<grid, block, smem_bytes, st>>>(p);
-            else k_run<P_AR, false><<<grid, block, smem_bytes, st>>>(p);
-            break;
-        default:
-            if (sm) k_run<P_AELL, true><<<grid, block, smem_bytes, st>>>(p);
-            else k_run<P_AELL, false><<<grid, block, smem_bytes, st>>>(p);
-            break;
+        case P_AMAX: launch_pol<P_AMAX>(p, grid, block, smem_bytes, st); break;
+        case P_AMIN: launch_pol<P_AMIN>(p, grid, block, smem_bytes, st); break;
+        case P_HSF: launch_pol<P_HSF>(p, grid, block, smem_bytes, st); break;
+        case P_AR: launch_pol<P_AR>(p, grid, block, smem_bytes, st); break;
+        default: launch_pol<P_AELL>(p, grid, block, smem_bytes, st); break;
     }
     return cudaGetLastError();
 }

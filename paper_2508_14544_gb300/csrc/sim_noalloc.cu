@@ -161,6 +161,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.lu = nullptr;
     p.tie_seed = nullptr;  // seed 0 for every instance, as sim_run without sim_set_tie_seeds
     p.work_count = nullptr;
+    p.batch_time = nullptr;
     p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
     p.dcap = kNaDeltaCap;
     p.use_smem = 0;

@@ -9,6 +9,8 @@
 //              Algorithm random, and the FIFO position 2 a for Algorithm promote_l, which also
 //              gets its (l, u) table).
 //   k_ratio  - per instance TEL(pi) / TEL(H-SF) in IEEE double (Definition cr).
+//   k_batch_time - per instance total latency and makespan in time units under a linear
+//              batch-time model (Section 6), from the integer sums the simulation recorded.
 #include <climits>
 #include <cstdint>
 
@@ -21,6 +23,10 @@ namespace {
 constexpr unsigned FULL = 0xffffffffu;
 enum { P_AMAX = 0, P_AMIN = 1, P_HSF = 2, P_AR = 3, P_AELL = 4 };
 enum { ST_OK = 0, ST_INVAL = -1, ST_INFEASIBLE = -2 };
+
+struct BtCoef {
+    double k[5];
+};
 
 __device__ __forceinline__ bool stage_less(int aa, const QEnt &x, int ab, const QEnt &y) {
     if (aa != ab) return aa < ab;
@@ -203,7 +209,43 @@ __global__ void k_ratio(const DevResult *pol, const DevResult *ref, double *out,
     out[i] = v;
 }
 
+// Total latency and makespan in time units under the linear batch-time model (Section 6: each
+// batch's time from a linear predictor; coef = c0, c1, c2, c3, c_idle):
+//   out[2i]     = c0 X0 + c1 X1 + c2 X2 + c3 X3,
+//   out[2i + 1] = c0 steps + c1 request_steps + c2 F2 + c3 F3 + c_idle (makespan - steps),
+// from sums = X0..X3, F2, F3 of instance i, evaluated left to right with round-to-nearest products
+// and sums (no fused multiply-add), so the result is the IEEE value of that expression.  NaN for an
+// instance that did not finish.
+__global__ void k_batch_time(const int64_t *sums, const DevResult *res, BtCoef c, double *out, int32_t n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const DevResult r = res[i];
+    const int64_t *x = sums + 6 * int64_t(i);
+    double tel = __longlong_as_double(0x7ff8000000000000ll), span = tel;
+    if (r.status == ST_OK) {
+        tel = __dadd_rn(__dadd_rn(__dadd_rn(__dmul_rn(c.k[0], __ll2double_rn(x[0])), __dmul_rn(c.k[1], __ll2double_rn(x[1]))),
+                                  __dmul_rn(c.k[2], __ll2double_rn(x[2]))),
+                        __dmul_rn(c.k[3], __ll2double_rn(x[3])));
+        span = __dadd_rn(__dadd_rn(__dadd_rn(__dadd_rn(__dmul_rn(c.k[0], __ll2double_rn(r.steps)),
+                                                       __dmul_rn(c.k[1], __ll2double_rn(r.request_steps))),
+                                             __dmul_rn(c.k[2], __ll2double_rn(x[4]))),
+                                   __dmul_rn(c.k[3], __ll2double_rn(x[5]))),
+                         __dmul_rn(c.k[4], __ll2double_rn(r.makespan - r.steps)));
+    }
+    out[2 * int64_t(i)] = tel;
+    out[2 * int64_t(i) + 1] = span;
+}
+
 }  // namespace
+
+cudaError_t launch_batch_time(const int64_t *sums, const DevResult *res, const double *coef, double *out, int32_t n,
+                              cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    BtCoef c;
+    for (int k = 0; k < 5; ++k) c.k[k] = coef[k];
+    k_batch_time<<<(n + 255) / 256, 256, 0, st>>>(sums, res, c, out, n);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
     if (p.n_inst <= 0) return cudaSuccess;

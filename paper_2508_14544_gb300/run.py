@@ -1,7 +1,7 @@
 """Command-line runner: simulate a named synthetic workload under one policy through the C ABI.
 
-  python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024] [--repeat 1]
-                                       [--warps-per-block W] [--warps-per-sm S]
+  python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024[:step]] [--repeat 1]
+                                       [--warps-per-block W] [--warps-per-sm S] [--evict-ties-by-index]
 
 Prints one JSON line per run with the wall time of sim_run, totals of the result fields, the
 throughput and a sha256 of the per-instance result records (equal across runs and launch shapes).
@@ -23,15 +23,15 @@ def main(argv=None) -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--workload", default="c2", choices=sorted(W.WORKLOADS))
     ap.add_argument("--policy", default="A_min", choices=sorted(POLICIES))
-    ap.add_argument("--instances", default=None, help="a:b range of instance ids (default: all)")
+    ap.add_argument("--instances", default=None, help="a:b or a:b:step range of instance ids (default: all)")
     ap.add_argument("--repeat", type=int, default=1)
     ap.add_argument("--warps-per-block", type=int, default=0)
     ap.add_argument("--warps-per-sm", type=int, default=0, help="residency limit (4: one warp per scheduler)")
+    ap.add_argument("--evict-ties-by-index", action="store_true", help="A_min: cancellation ties by index")
     args = ap.parse_args(argv)
     ids = None
     if args.instances:
-        a, b = (int(x) for x in args.instances.split(":"))
-        ids = range(a, b)
+        ids = range(*(int(x) for x in args.instances.split(":")))
     w = W.make_workload(args.workload, ids)
     import torch
     dev = [torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (w.arrival, w.prompt, w.lower, w.upper, w.true_o)]
@@ -41,6 +41,8 @@ def main(argv=None) -> None:
         opts["warps_per_block"] = args.warps_per_block
     if args.warps_per_sm:
         opts["warps_per_sm"] = args.warps_per_sm
+    if args.evict_ties_by_index:
+        opts["evict_ties"] = 1
     with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
         sim.set_tie_seeds(w.tie_seeds())
         for _ in range(args.repeat):
@@ -56,7 +58,8 @@ def main(argv=None) -> None:
                               "request_steps_per_s": rs / dt, "steps_per_s": st / dt,
                               "total_latency": int(res["total_latency"].sum()),
                               "evictions": int(res["evictions"].sum()),
-                              "most_evictions": [int(ids[0] if ids else 0) + int(np.argmax(res["evictions"])),
+                              "most_evictions": [int(ids[int(np.argmax(res["evictions"]))]) if ids else
+                                                 int(np.argmax(res["evictions"])),
                                                  int(res["evictions"].max())],
                               "worst_status": int(res["status"].min()), "results_sha256": digest}), flush=True)
 

@@ -24,7 +24,7 @@ class Simulator:
                "warps_per_block": L.SIM_OPT_WARPS_PER_BLOCK, "smem_active_cap": L.SIM_OPT_SMEM_ACTIVE_CAP,
                "warps_per_sm": L.SIM_OPT_WARPS_PER_SM, "debug_checks": L.SIM_OPT_DEBUG_CHECKS,
                "tune_residency": L.SIM_OPT_TUNE_RESIDENCY, "evict_ties": L.SIM_OPT_EVICT_TIES,
-               "count_work": L.SIM_OPT_COUNT_WORK}
+               "count_work": L.SIM_OPT_COUNT_WORK, "batch_time": L.SIM_OPT_BATCH_TIME}
 
     def set_option(self, name: str, value: int) -> None:
         rc = L.sim_set_option(self.ctx, self.OPTIONS[name], int(value))
@@ -77,6 +77,19 @@ class Simulator:
         out = np.zeros(4 * self.n_instances, dtype=np.int64)
         self._check(L.sim_get_work_counts(self.ctx, out))
         return out.reshape(self.n_instances, 4)
+
+    def batch_time(self, coef, stream: int = 0) -> np.ndarray:
+        """[n_instances, 2] (total latency, makespan) in time units under the linear batch-time
+        model coef = (c0, c1, c2, c3, c_idle) (option batch_time=1 for the last run)."""
+        out = np.zeros(2 * self.n_instances, dtype=np.float64)
+        self._check(L.sim_batch_time(self.ctx, coef, out, stream))
+        return out.reshape(self.n_instances, 2)
+
+    def batch_time_sums(self) -> np.ndarray:
+        """[n_instances, 6] int64: X0..X3, F2, F3 of the last run (option batch_time=1)."""
+        out = np.zeros(6 * self.n_instances, dtype=np.int64)
+        self._check(L.sim_get_batch_time_sums(self.ctx, out))
+        return out.reshape(self.n_instances, 6)
 
     def completions(self, n_total: int) -> np.ndarray:
         out = np.zeros(max(n_total, 1), dtype=np.int64)
