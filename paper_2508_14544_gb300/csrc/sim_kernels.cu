@@ -255,6 +255,35 @@ __device__ __forceinline__ int lane_prefix_count(int len, Pred pred) {
     return lo;
 }
 
+// Position of the job A_min cancels when several live jobs (F >= 0) of the active set share the
+// smallest estimate mk: the smallest (tie key, index) among them, the tie key drawn from `base`
+// (tie_base of the step) or, under the index rule, the index itself.  Warp-wide; every lane gets
+// the position.  Out of line: ties are a small share of the cancellation rounds, and keeping the
+// hashing out of the simulation loop keeps that loop's code small (the loop is sensitive to the
+// instruction cache).
+__device__ __noinline__ int tie_position(const int32_t *F, const int32_t *K, const int32_t *I, int A, unsigned mk,
+                                         uint64_t base, int rnd) {
+    const int lane = lane_id();
+    unsigned br = UINT_MAX, bi = UINT_MAX;
+    int bp = -1;
+    #pragma unroll 1
+    for (int i = lane; i < A; i += 32) {
+        if (F[i] >= 0 && unsigned(K[i]) == mk) {
+            const unsigned id = unsigned(I[i]);
+            const unsigned r = rnd ? tie_key(base, int(id)) : id;
+            if (r < br || (r == br && id < bi)) {
+                br = r;
+                bi = id;
+                bp = i;
+            }
+        }
+    }
+    const unsigned mr = __reduce_min_sync(FULL, br);
+    const unsigned mi = __reduce_min_sync(FULL, br == mr ? bi : UINT_MAX);
+    const unsigned b = __ballot_sync(FULL, bp >= 0 && br == mr && bi == mi);
+    return b ? __shfl_sync(FULL, bp, __ffs(b) - 1) : -1;
+}
+
 // ---------------------------------------------------------------------------------------------
 // Per-warp workspace
 // ---------------------------------------------------------------------------------------------
@@ -314,17 +343,17 @@ struct Queue {
     int mbuf;        // -1: mq is read-only staged data; 0/1: ping-pong buffer in use
     int dn;          // delta size
     int mcb;         // main cache base: w.mc[i] = mq[mcb + i] for i < kMc; -1 invalid
-    int64_t gb;      // global-memory bytes the queue has moved (work counter)
 };
 
 __device__ __forceinline__ bool queue_empty(const Queue &q) { return q.mh >= q.me && q.dn == 0; }
 
 // Make w.mc cover mq[mh .. mh + kWin): keep the cached run while the head is within its first
-// kMc - kWin entries, otherwise reload kMc entries from the head.
-__device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
+// kMc - kWin entries, otherwise reload kMc entries from the head.  gb counts the global-memory bytes
+// the queue moves (a work counter of the instrumented kernel; a dead variable otherwise).
+__device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q, int64_t &gb) {
     if (q.mcb >= 0 && q.mh >= q.mcb && q.mh - q.mcb <= kMc - kWin) return;
     const int lane = lane_id();
-    q.gb += int64_t(min(kMc, q.me - q.mh)) * int64_t(sizeof(QEnt));
+    gb += int64_t(min(kMc, q.me - q.mh)) * int64_t(sizeof(QEnt));
     const int i0 = q.mh + lane, i1 = q.mh + 32 + lane;
     QEnt a, b;
     if (i0 < q.me) a = q.mq[i0];
@@ -338,8 +367,8 @@ __device__ __forceinline__ void main_cache_at_head(const Ws &w, Queue &q) {
 // Merge the delta into the main array (into the other ping-pong buffer).  Rare (a full delta, or
 // a long arrival run), so it is kept out of line: the simulation loop stays small enough for the
 // instruction cache when two warps share a scheduler.  Takes the few workspace pointers it needs
-// by value and the queue by pointer.
-__device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0, QEnt *mb1, Queue *qp) {
+// by value and the queue by pointer; gb (null in the plain kernel) counts the global bytes moved.
+__device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0, QEnt *mb1, Queue *qp, int64_t *gb) {
     const int lane = lane_id();
     Queue q = *qp;
     const int dn = q.dn;
@@ -389,7 +418,7 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
     }
     __syncwarp();
     __threadfence_block();
-    q.gb += int64_t(2 * nx + dn) * int64_t(sizeof(QEnt));  // main read once, merged array written
+    if (gb && lane == 0) *gb += int64_t(2 * nx + dn) * int64_t(sizeof(QEnt));  // main read once, merged written
     q.mq = out;
     q.mbuf = (q.mbuf == 0) ? 1 : 0;
     q.mh = 0;
@@ -399,16 +428,16 @@ __device__ __noinline__ void merge_delta(int32_t *cnt, const QEnt *dq, QEnt *mb0
     *qp = q;
 }
 
-__device__ __forceinline__ void merge_delta(const Ws &w, Queue &q) {
+__device__ __forceinline__ void merge_delta(const Ws &w, Queue &q, int64_t *gb) {
     Queue qq = q;
-    merge_delta(w.cnt, w.dq, w.mb0, w.mb1, &qq);
+    merge_delta(w.cnt, w.dq, w.mb0, w.mb1, &qq, gb);
     q = qq;
 }
 
 // Insert one entry into the delta (merging the delta into main first if it is full).
-__device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &e) {
+__device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &e, int64_t *gb) {
     const int lane = lane_id();
-    if (q.dn == w.dcap) merge_delta(w, q);
+    if (q.dn == w.dcap) merge_delta(w, q, gb);
     const int dn = q.dn;
     if (dn < 64) {
         // two entries per lane: count the entries greater than e (they lead the descending delta),
@@ -444,11 +473,11 @@ __device__ __forceinline__ void delta_insert(const Ws &w, Queue &q, const QEnt &
 }
 
 // Head of R_t (smallest (key, idx)); the queue must not be empty.
-__device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q) {
+__device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q, int64_t &gb) {
     const bool have_m = q.mh < q.me;
     QEnt hm;
     if (have_m) {
-        main_cache_at_head(w, q);
+        main_cache_at_head(w, q, gb);
         hm = w.mc[q.mh - q.mcb];
     }
     if (q.dn > 0) {
@@ -460,10 +489,11 @@ __device__ __forceinline__ QEnt queue_head(const Ws &w, Queue &q) {
 
 // Arrival batch (ascending run in global memory): becomes the main array if R_t is empty; a few
 // entries go into the delta one by one; a long batch is copied into the emptied delta in chunks.
-__device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len) {
+__device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *run, int len, int64_t &gb,
+                                           int64_t *gbp) {
     const int lane = lane_id();
     if (len <= 0) return;
-    q.gb += int64_t(len) * int64_t(sizeof(QEnt));
+    gb += int64_t(len) * int64_t(sizeof(QEnt));
     if (queue_empty(q)) {
         q.mq = run;
         q.mh = 0;
@@ -478,10 +508,10 @@ __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *ru
         const int rem = len - done;
         if (rem <= 8) {
             #pragma unroll 1
-            for (int j = 0; j < rem; ++j) delta_insert(w, q, run[done + j]);
+            for (int j = 0; j < rem; ++j) delta_insert(w, q, run[done + j], gbp);
             break;
         }
-        if (q.dn > 0) merge_delta(w, q);
+        if (q.dn > 0) merge_delta(w, q, gbp);
         const int k = min(rem, w.dcap);
         #pragma unroll 1
         for (int j = lane; j < k; j += 32) w.dq[j] = run[done + k - 1 - j];  // descending
@@ -494,10 +524,10 @@ __device__ __forceinline__ void insert_run(const Ws &w, Queue &q, const QEnt *ru
 // First kWin entries of R_t in (key, idx) order from the cached head of the main array (ascending)
 // and the delta (descending): lane m returns entry m in `mine` (src 0 main, 1 delta).  Returns how
 // many there are.
-__device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, int &msrc) {
+__device__ __forceinline__ int build_window(const Ws &w, Queue &q, QEnt &mine, int &msrc, int64_t &gb) {
     const int lane = lane_id();
     const int nmain = max(q.me - q.mh, 0);
-    if (nmain > 0) main_cache_at_head(w, q);
+    if (nmain > 0) main_cache_at_head(w, q, gb);
     const int na = min(kWin, nmain);
     const int dn = q.dn;
     const int nb = min(kWin, dn);
@@ -1137,9 +1167,6 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     const QEnt *rec = P.rec + info.base;
     const int32_t *ra = P.rec_a + info.base;
     const uint64_t tie_seed = (POL == P_AMIN && P.tie_seed) ? P.tie_seed[inst] : 0ull;
-    // bits of the longest length (every A_min estimate is below 2^kbits), for the packed
-    // cancellation keys
-    const int kbits = 32 - __clz(max(info.lmax, 1));
     const int64_t M = P.M;
     const int64_t cap = info.cap;
 
@@ -1149,7 +1176,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     q.mbuf = -1;
     q.dn = 0;
     q.mcb = -1;
-    q.gb = 0;
+    // global-memory bytes moved by the queue (instrumented kernel); the merge adds through gbp
+    int64_t gbq = 0;
+    int64_t *const gbp = INS ? &gbq : nullptr;
     // work counters of the paper's per-step method (Theorem complexity), accumulated per step in
     // closed form: S2 adds (the active set), S3 compare-exchanges of the overflow sort
     // (A ceil(log2 A)^2), S5 endpoint evaluations of a binary-search admission
@@ -1229,8 +1258,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 ae += k;
                 if (k < 32) break;
             }
-            insert_run(w, q, rec + ap, ae - ap);
-            if (INS) q.gb += int64_t(ae - ap) * 4;  // their arrival steps
+            insert_run(w, q, rec + ap, ae - ap, gbq, gbp);
+            if (INS) gbq += int64_t(ae - ap) * 4;  // their arrival steps
             if (bt) {
                 const int64_t m = ae - ap;
                 bx0 -= m * steps;
@@ -1259,75 +1288,43 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     cS3 += int64_t(A) * lg * lg;
                 }
                 // Cancellation order (estimate, r, index), r the step's tie key (SplitMix64 of the seed
-                // and t * 2^32 + index; under the index rule r = index, the same order).
-                const uint64_t tb64 = tie_base(tie_seed, t);
-                const bool rnd = P.evict_index == 0;
-                // One-chunk sets: the lane's four entries are keyed once per step, in registers, by
-                // pk = estimate << (32 - kb) | r >> kb (estimate < 2^kb), whose order is that of
-                // (estimate, high bits of r); a round takes one warp minimum of pk, and only equal pk
-                // (the same estimate and the same high bits of r) look at all of r, then the index.
-                // A cancelled or missing entry holds pk = UINT_MAX and is never a candidate.
+                // and t * 2^32 + index; under the index rule r = index, the same order).  A round
+                // finds the smallest estimate by one warp minimum; only when several live jobs share
+                // it does tie_position draw and compare their keys.  (On the 40960 x 2000 workload
+                // 1.3 % of the overflow steps have a tie at the smallest estimate.)
+                // One-chunk sets keep the lane's four estimates in registers for all of the step's
+                // cancellations, `live` marking those still in the set (the array itself is never
+                // written by a run-time position, which would put it in local memory).
                 const bool reg = A <= kChunk;
-                unsigned pk[4] = {UINT_MAX, UINT_MAX, UINT_MAX, UINT_MAX}, rr[4] = {0u, 0u, 0u, 0u};
-                int ri[4] = {0, 0, 0, 0};
-                unsigned live = 0;  // bit j: entry j of the lane is a live job
+                unsigned rk[4] = {0u, 0u, 0u, 0u};
+                unsigned live = 0;
                 if (reg) {
                     const int base = 4 * lane;
-                    const int4 k4 = ld4(w.K, base), i4 = ld4(w.I, base);
-                    const int kk[4] = {k4.x, k4.y, k4.z, k4.w}, ii[4] = {i4.x, i4.y, i4.z, i4.w};
+                    const int4 k4 = ld4(w.K, base);
+                    const int kk[4] = {k4.x, k4.y, k4.z, k4.w};
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        ri[j] = ii[j];
-                        if (base + j < A) {
-                            live |= 1u << j;
-                            rr[j] = rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]);
-                            pk[j] = (unsigned(kk[j]) << (32 - kbits)) | (kbits == 32 ? 0u : rr[j] >> kbits);
-                        }
+                        rk[j] = unsigned(kk[j]);
+                        if (base + j < A) live |= 1u << j;
                     }
                 }
                 #pragma unroll 1
                 while (need > wint<N>(M)) {
                     int pos = -1;
+                    unsigned mk;
+                    int tot = 0;
                     if (reg) {
-                        const unsigned mk = __reduce_min_sync(FULL, min(min(pk[0], pk[1]), min(pk[2], pk[3])));
-                        unsigned cand = 0;  // bit j: entry j holds the smallest packed key
-                        int tot = 0;
+                        const unsigned q0 = (live & 1u) ? rk[0] : UINT_MAX, q1 = (live & 2u) ? rk[1] : UINT_MAX;
+                        const unsigned q2 = (live & 4u) ? rk[2] : UINT_MAX, q3 = (live & 8u) ? rk[3] : UINT_MAX;
+                        mk = __reduce_min_sync(FULL, min(min(q0, q1), min(q2, q3)));
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
-                            const bool c = ((live >> j) & 1u) && pk[j] == mk;
-                            cand |= c ? (1u << j) : 0u;
-                            const unsigned b = __ballot_sync(FULL, c);
+                            const unsigned b = __ballot_sync(FULL, ((live >> j) & 1u) && rk[j] == mk);
                             tot += __popc(b);
                             if (b) pos = 4 * (__ffs(b) - 1) + j;
                         }
-                        if (tot > 1) {  // equal packed keys: all of r, then the index
-                            unsigned lr = UINT_MAX;
-#pragma unroll
-                            for (int j = 0; j < 4; ++j)
-                                if ((cand >> j) & 1u) lr = min(lr, rr[j]);
-                            const unsigned mr = __reduce_min_sync(FULL, lr);
-                            unsigned li = UINT_MAX;
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                if (rr[j] != mr) cand &= ~(1u << j);
-                                if ((cand >> j) & 1u) li = min(li, unsigned(ri[j]));
-                            }
-                            const unsigned mi = __reduce_min_sync(FULL, li);
-#pragma unroll
-                            for (int j = 0; j < 4; ++j) {
-                                const unsigned b = __ballot_sync(FULL, ((cand >> j) & 1u) && unsigned(ri[j]) == mi);
-                                if (b) pos = 4 * (__ffs(b) - 1) + j;
-                            }
-                        }
-                        if (pos >= 0 && (pos >> 2) == lane) {
-#pragma unroll
-                            for (int j = 0; j < 4; ++j)
-                                if ((pos & 3) == j) pk[j] = UINT_MAX;
-                            live &= ~(1u << (pos & 3));
-                        }
                     } else {
-                        // wider sets: one pass for the smallest estimate, how many live jobs share it
-                        // and (if one) where; a second pass draws the tied jobs' keys otherwise
+                        // one pass: the smallest estimate, how many live jobs share it, and where
                         unsigned bk = UINT_MAX;
                         int bc = 0, bp = -1;
                         #pragma unroll 1
@@ -1349,38 +1346,14 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                                 }
                             }
                         }
-                        const unsigned mk = __reduce_min_sync(FULL, bk);
-                        const int tot = int(__reduce_add_sync(FULL, bk == mk ? unsigned(bc) : 0u));
-                        if (mk != UINT_MAX && tot == 1) {
-                            const unsigned b = __ballot_sync(FULL, bk == mk && bc > 0);
-                            pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
-                        } else if (mk != UINT_MAX) {
-                            unsigned br = UINT_MAX, bi = UINT_MAX;
-                            bp = -1;
-                            #pragma unroll 1
-                            for (int cb = 0; cb < A; cb += kChunk) {
-                                const int base = cb + 4 * lane;
-                                const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base), i4 = ld4(w.I, base);
-                                const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
-                                const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
-#pragma unroll
-                                for (int j = 0; j < 4; ++j) {
-                                    if (base + j < A && ff[j] >= 0 && unsigned(kk[j]) == mk) {
-                                        const unsigned r = rnd ? tie_key(tb64, ii[j]) : unsigned(ii[j]);
-                                        if (r < br || (r == br && unsigned(ii[j]) < bi)) {
-                                            br = r;
-                                            bi = unsigned(ii[j]);
-                                            bp = base + j;
-                                        }
-                                    }
-                                }
-                            }
-                            const unsigned mr = __reduce_min_sync(FULL, br);
-                            const unsigned mi = __reduce_min_sync(FULL, br == mr ? bi : UINT_MAX);
-                            const unsigned b = __ballot_sync(FULL, bp >= 0 && br == mr && bi == mi);
-                            pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
-                        }
+                        mk = __reduce_min_sync(FULL, bk);
+                        tot = int(__reduce_add_sync(FULL, bk == mk ? unsigned(bc) : 0u));
+                        const unsigned b = __ballot_sync(FULL, bk == mk && bc > 0);
+                        if (b) pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
                     }
+                    if (mk == UINT_MAX) pos = -1;
+                    else if (tot > 1) pos = tie_position(w.F, w.K, w.I, A, mk, tie_base(tie_seed, t), P.evict_index == 0);
+                    if (reg && pos >= 0 && (pos >> 2) == lane) live &= ~(1u << (pos & 3));
                     if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
                         break;
@@ -1397,7 +1370,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     need -= wint<N>(b) + t;
                     ++nev;
                     if (INS) ++ev_step;
-                    delta_insert(w, q, e);
+                    delta_insert(w, q, e, gbp);
                 }
                 if (status != ST_OK) break;
                 tb_next = t;
@@ -1425,7 +1398,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 __syncwarp();
                 if (lane == 0) w.F[j] = -1;
                 __syncwarp();
-                delta_insert(w, q, e);
+                delta_insert(w, q, e, gbp);
             }
             nev += c;
             if (INS) ev_step += c;
@@ -1438,7 +1411,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
         for (;;) {
             if (!hvalid) {
                 if (queue_empty(q)) break;
-                h = proj<POL>(P, info.base, queue_head(w, q));
+                h = proj<POL>(P, info.base, queue_head(w, q, gbq));
                 hvalid = true;
                 pdirty = true;
             }
@@ -1469,7 +1442,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             QEnt mine;
             mine.key = mine.idx = mine.s = mine.o = 0;
             int msrc = 0;
-            const int W = build_window(w, q, mine, msrc);
+            const int W = build_window(w, q, mine, msrc, gbq);
             if (POL == P_AR || POL == P_AELL) {
                 if (lane < W) mine = proj<POL>(P, info.base, mine);
             }
@@ -1593,7 +1566,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             wc[0] = cS2;
             wc[1] = cS3;
             wc[2] = cS5;
-            wc[3] = q.gb;
+            wc[3] = gbq;
         }
     }
     __syncwarp();
