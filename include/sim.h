@@ -102,15 +102,17 @@ enum {
                                        H-SF and A_r).  A violation gives that instance SIM_E_STATE.
                                        Slower; results are otherwise identical. */
     SIM_OPT_TUNE_RESIDENCY = 7,     /* 0/1: on the first sim_run of a load shape (n_instances, total
-                                       and largest instance size), time the simulation launch with
-                                       one warp per scheduler (4 per SM) and with the default
-                                       residency, and use the faster for every later sim_run of
-                                       that shape, across sim_load calls (default 0).  A launch is
-                                       as long as its slowest instance: one warp per scheduler
-                                       wins when a few instances dominate (A_min with long
-                                       cancellation chains), two when instances are even.  The
-                                       tuning run simulates twice; results do not depend on it.
-                                       Overrides SIM_OPT_WARPS_PER_SM while set. */
+                                       and largest instance size), time three residencies -- one
+                                       simulation warp per scheduler (4 per SM), the default (two),
+                                       and the dense configuration of SIM_OPT_DENSE_RESIDENCY
+                                       (three) -- each with its global-memory re-runs, and use the
+                                       fastest for every later sim_run of that shape, across
+                                       sim_load calls (default 0).  A launch is as long as its
+                                       slowest instance: one warp per scheduler wins when a few
+                                       instances dominate, more when there are many even ones.  The
+                                       tuning run simulates three times; results do not depend on
+                                       it.  Overrides SIM_OPT_WARPS_PER_SM and
+                                       SIM_OPT_DENSE_RESIDENCY while set. */
     SIM_OPT_EVICT_TIES = 8,         /* 0 (default): A_min's cancellation ties are broken at random
                                        as Algorithm milb states (see sim_set_tie_seeds); 1: by the
                                        request index instead, a fixed order that always cancels the
@@ -118,9 +120,17 @@ enum {
     SIM_OPT_COUNT_WORK = 9,         /* 0/1: record per instance the work that the paper's per-step
                                        method does (sim_get_work_counts; default 0).  Results are
                                        identical; the counting costs a few instructions per event. */
-    SIM_OPT_BATCH_TIME = 10         /* 0/1: record per instance the integer sums that give total
+    SIM_OPT_BATCH_TIME = 10,        /* 0/1: record per instance the integer sums that give total
                                        latency and makespan in time units under a linear batch-time
                                        model (sim_batch_time, sim_get_batch_time_sums; default 0). */
+    SIM_OPT_DENSE_RESIDENCY = 11    /* 0/1: simulate with three blocks of four warps per SM (12
+                                       warps; a kernel copy limited to 170 registers a thread) and
+                                       384 active-set slots in shared memory per instance, instead
+                                       of two blocks and SIM_OPT_SMEM_ACTIVE_CAP slots (default 0).
+                                       Faster when there are many instances whose active sets stay
+                                       below 384 jobs; instances that need more are re-run in global
+                                       memory.  Not used with SIM_OPT_COUNT_WORK or
+                                       SIM_OPT_BATCH_TIME.  Results do not depend on it. */
 };
 
 /*

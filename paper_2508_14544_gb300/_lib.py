@@ -22,6 +22,7 @@ SIM_OPT_TUNE_RESIDENCY = 7
 SIM_OPT_EVICT_TIES = 8
 SIM_OPT_COUNT_WORK = 9
 SIM_OPT_BATCH_TIME = 10
+SIM_OPT_DENSE_RESIDENCY = 11
 
 STATUS_NAMES = {0: "SIM_OK", -1: "SIM_E_INVAL", -2: "SIM_E_INFEASIBLE", -3: "SIM_E_STEPCAP", -4: "SIM_E_CUDA",
                 -5: "SIM_E_STATE", -6: "SIM_E_NOMEM"}

@@ -31,12 +31,14 @@ struct sim_ctx {
     int warps_per_sm = 0;
     int debug_checks = 0;
     int tune_residency = 0;
+    int dense = 0;  // SIM_OPT_DENSE_RESIDENCY
     int evict_index = 0;
     int count_work = 0;
     int batch_time = 0;
     // residency chosen by SIM_OPT_TUNE_RESIDENCY for the load shape tuned_shape (n_inst, n_total,
     // n_max): warps per SM, or 0 for the default; tuned_shape[0] < 0 when not tuned
     int tuned_wps = 0;
+    int tuned_dense = 0;
     int64_t tuned_shape[3] = {-1, -1, -1};
     int smem_ca = 512;
     int dcap = 256;
@@ -182,6 +184,9 @@ int sim_set_option(sim_ctx *c, int key, int64_t value) {
             if (value != 0 && value != 1) return fail(c, SIM_E_INVAL, "EVICT_TIES must be 0 (random) or 1 (index)");
             c->evict_index = int(value);
             return SIM_OK;
+        case SIM_OPT_DENSE_RESIDENCY:
+            c->dense = value ? 1 : 0;
+            return SIM_OK;
         case SIM_OPT_COUNT_WORK:
             c->count_work = value ? 1 : 0;
             return SIM_OK;
@@ -319,16 +324,21 @@ int sim_load(sim_ctx *c, int32_t n, const int32_t *a, const int32_t *s, const in
     return sim_load_csr(c, off.data(), a, s, l, u, o, device_ptrs);
 }
 
+// One launch of the simulation kernel over n_work instances (all, or the device list work_dev).
+// smem: the active sets in shared memory (else a global-memory workspace of n_max slots);
+// dense: the 12-warps-per-SM configuration (blocks of 4 warps, 384 shared-memory slots); not with
+// the instrumented kernel, which keeps its own register budget.
 static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int32_t n_work, bool smem,
-                      int warps_per_sm) {
+                      int warps_per_sm, bool dense = false) {
     cudaError_t e;
     int dev = c->device;
     int n_sm = 0, smem_optin = 0;
     cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
     cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    int wpb = c->wpb;
+    dense = dense && smem && !c->count_work && !c->batch_time;
+    int wpb = dense ? simgb::kDenseWarps : c->wpb;
     const int dcap = c->dcap;
-    int ca = smem ? c->smem_ca : ((std::max(c->n_max, 128) + 127) / 128) * 128;
+    int ca = smem ? (dense ? simgb::kDenseCa : c->smem_ca) : ((std::max(c->n_max, 128) + 127) / 128) * 128;
     size_t per_warp = simgb::warp_ws_bytes(ca, dcap);
     size_t smem_bytes = 0;
     if (smem) {
@@ -343,11 +353,11 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
         int smem_sm = 0;
         cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
         per_sm = std::max(1, int(size_t(smem_sm) / (smem_bytes + 1024)));
-        per_sm = std::min(per_sm, 64 / wpb);
+        per_sm = std::min(per_sm, dense ? 3 : 64 / wpb);
     } else {
         per_sm = std::max(1, 16 / wpb);
     }
-    if (warps_per_sm > 0) per_sm = std::max(1, std::min(per_sm, warps_per_sm / wpb));
+    if (warps_per_sm > 0 && !dense) per_sm = std::max(1, std::min(per_sm, warps_per_sm / wpb));
     int64_t blocks = int64_t(n_sm) * per_sm;
     blocks = std::min<int64_t>(blocks, (n_work + wpb - 1) / wpb);
     blocks = std::max<int64_t>(blocks, 1);
@@ -396,10 +406,56 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.main_cap = main_cap;
     if ((e = cudaMemsetAsync(c->d_counter, 0, sizeof(int32_t), st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaMemsetAsync");
-    e = simgb::launch_run(c->policy, p, int(blocks), wpb, smem_bytes, st);
+    e = simgb::launch_run(c->policy, p, int(blocks), wpb, smem_bytes, dense, st);
     if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: kernel launch");
     ++c->launches;
     return SIM_OK;
+}
+
+// Simulate every instance (shared-memory kernel, then a global-memory re-run of the instances whose
+// active set outgrew it) and copy the results to c->h_res; ms (optional) receives the device time
+// of the whole, measured by events on the stream.
+static int simulate(sim_ctx *c, cudaStream_t st, int wps, bool dense, float *ms) {
+    cudaError_t e;
+    cudaEvent_t ev[2] = {nullptr, nullptr};
+    if (ms) {
+        for (auto &x : ev)
+            if ((e = cudaEventCreate(&x)) != cudaSuccess) return cuda_fail(c, e, "cudaEventCreate");
+        cudaEventRecord(ev[0], st);
+    }
+    int rc = run_launch(c, st, nullptr, c->n_inst, !c->debug_checks, wps, dense);
+    if (rc == SIM_OK) {
+        c->h_res.resize(size_t(c->n_inst));
+        e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost,
+                            st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) rc = cuda_fail(c, e, "sim_run: simulation kernel");
+    }
+    // instances whose active set outgrew the shared-memory workspace: re-run from global memory
+    std::vector<int32_t> redo;
+    if (rc == SIM_OK)
+        for (int32_t i = 0; i < c->n_inst; ++i)
+            if (c->h_res[i].status == simgb::kStatusCapacity) redo.push_back(i);
+    if (rc == SIM_OK && !redo.empty()) {
+        e = cudaMemcpyAsync(c->d_work, redo.data(), redo.size() * sizeof(int32_t), cudaMemcpyHostToDevice, st);
+        if (e != cudaSuccess) rc = cuda_fail(c, e, "sim_run: work list");
+        if (rc == SIM_OK) rc = run_launch(c, st, c->d_work, int32_t(redo.size()), false, c->warps_per_sm);
+        if (rc == SIM_OK) {
+            e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst),
+                                cudaMemcpyDeviceToHost, st);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+            if (e != cudaSuccess) rc = cuda_fail(c, e, "sim_run: simulation kernel (global workspace)");
+        }
+    }
+    if (ms) {
+        if (rc == SIM_OK) {
+            cudaEventRecord(ev[1], st);
+            if ((e = cudaEventSynchronize(ev[1])) == cudaSuccess) cudaEventElapsedTime(ms, ev[0], ev[1]);
+            else rc = cuda_fail(c, e, "sim_run: residency tuning");
+        }
+        for (auto &x : ev) cudaEventDestroy(x);
+    }
+    return rc;
 }
 
 int sim_run(sim_ctx *c, sim_result *out, void *stream) {
@@ -431,57 +487,37 @@ int sim_run(sim_ctx *c, sim_result *out, void *stream) {
     }
     // with SIM_OPT_DEBUG_CHECKS every instance runs in the checking global-memory kernel
     int wps = c->warps_per_sm;
-    bool simulated = false;  // a tuning launch already wrote the results (they do not depend on residency)
+    bool dense = c->dense != 0;
+    bool simulated = false;  // a tuning run already wrote the results (they do not depend on residency)
     if (c->tune_residency && !c->debug_checks) {
         const int64_t shape[3] = {c->n_inst, c->n_total, c->n_max};
         if (!std::equal(shape, shape + 3, c->tuned_shape)) {
-            // one warp per scheduler (4 schedulers per SM) against the default, timed on the stream
-            cudaEvent_t ev[3];
-            for (auto &x : ev)
-                if ((e = cudaEventCreate(&x)) != cudaSuccess) return cuda_fail(c, e, "cudaEventCreate");
-            const int cand[2] = {4, 0};
-            float ms[2] = {0.f, 0.f};
-            cudaEventRecord(ev[0], st);
-            for (int k = 0; k < 2 && rc == SIM_OK; ++k) {
-                rc = run_launch(c, st, nullptr, c->n_inst, true, cand[k]);
-                cudaEventRecord(ev[k + 1], st);
+            // one warp per scheduler (4 schedulers per SM), the default (two), and the dense copy
+            // (three), each timed on the stream with its capacity re-runs
+            const int cand_wps[3] = {4, 0, 0};
+            const bool cand_dense[3] = {false, false, true};
+            float best = 0.f;
+            int pick = 1;
+            for (int k = 0; k < 3; ++k) {
+                float ms = 0.f;
+                rc = simulate(c, st, cand_wps[k], cand_dense[k], &ms);
+                if (rc) return rc;
+                if (k == 0 || ms < best) {
+                    best = ms;
+                    pick = k;
+                }
             }
-            if (rc == SIM_OK && (e = cudaEventSynchronize(ev[2])) == cudaSuccess) {
-                cudaEventElapsedTime(&ms[0], ev[0], ev[1]);
-                cudaEventElapsedTime(&ms[1], ev[1], ev[2]);
-                c->tuned_wps = ms[0] < ms[1] ? cand[0] : cand[1];
-                std::copy(shape, shape + 3, c->tuned_shape);
-                simulated = true;
-            }
-            for (auto &x : ev) cudaEventDestroy(x);
-            if (rc) return rc;
-            if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: residency tuning");
+            c->tuned_wps = cand_wps[pick];
+            c->tuned_dense = cand_dense[pick] ? 1 : 0;
+            std::copy(shape, shape + 3, c->tuned_shape);
+            simulated = true;
         }
         wps = c->tuned_wps;
+        dense = c->tuned_dense != 0;
     }
     if (!simulated) {
-        rc = run_launch(c, st, nullptr, c->n_inst, !c->debug_checks, wps);
+        rc = simulate(c, st, wps, dense && !c->debug_checks, nullptr);
         if (rc) return rc;
-    }
-    c->h_res.resize(size_t(c->n_inst));
-    e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost, st);
-    if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: copy of the results");
-    e = cudaStreamSynchronize(st);
-    if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: simulation kernel");
-    // instances whose active set outgrew the shared-memory workspace: re-run from global memory
-    std::vector<int32_t> redo;
-    for (int32_t i = 0; i < c->n_inst; ++i)
-        if (c->h_res[i].status == simgb::kStatusCapacity) redo.push_back(i);
-    if (!redo.empty()) {
-        e = cudaMemcpyAsync(c->d_work, redo.data(), redo.size() * sizeof(int32_t), cudaMemcpyHostToDevice, st);
-        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: work list");
-        rc = run_launch(c, st, c->d_work, int32_t(redo.size()), false, c->warps_per_sm);
-        if (rc) return rc;
-        e = cudaMemcpyAsync(c->h_res.data(), c->d_res, sizeof(DevResult) * size_t(c->n_inst), cudaMemcpyDeviceToHost,
-                            st);
-        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: copy of the results");
-        e = cudaStreamSynchronize(st);
-        if (e != cudaSuccess) return cuda_fail(c, e, "sim_run: simulation kernel (global workspace)");
     }
     int worst = SIM_OK;
     for (int32_t i = 0; i < c->n_inst; ++i) {

@@ -90,8 +90,11 @@ struct RunParams {
 size_t warp_ws_bytes(int ca, int dcap);
 
 cudaError_t launch_stage(const StageParams &p, cudaStream_t st);
-cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
+// dense: the 12-warps-per-SM copy of the plain shared-memory kernel (blocks of 4 warps)
+cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes, bool dense,
                        cudaStream_t st);
+constexpr int kDenseCa = 384;      // active-set slots per warp of the dense configuration
+constexpr int kDenseWarps = 4;     // warps per block of the dense configuration
 cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
 cudaError_t launch_batch_time(const int64_t *sums, const DevResult *res, const double *coef, double *out, int32_t n,
                               cudaStream_t st);

@@ -1,4 +1,4 @@
-// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared, instrumented>.
+// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared, instrumented, dense>.
 //
 // One warp simulates one instance at a time (persistent warps pull instance ids from a work
 // queue).  Each step follows the paper's algorithms:
@@ -1572,8 +1572,11 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     __syncwarp();
 }
 
-template <int POL, bool SMEM, bool INS>
-__global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
+// DENSE: the copy for three blocks of four warps per SM (12 simulating warps, at most 170
+// registers a thread), which the host pairs with a 384-slot shared-memory active set; otherwise
+// blocks of up to 256 threads and as many registers as the code wants (two blocks per SM).
+template <int POL, bool SMEM, bool INS, bool DENSE>
+__global__ void __launch_bounds__(DENSE ? 128 : 256, DENSE ? 3 : 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
     const int wib = threadIdx.x >> 5;
@@ -1595,21 +1598,24 @@ __global__ void __launch_bounds__(256, 1) k_run(RunParams P) {
 }
 
 template <int POL>
-const void *run_fn(bool smem, bool ins) {
-    if (ins) return smem ? (const void *)k_run<POL, true, true> : (const void *)k_run<POL, false, true>;
-    return smem ? (const void *)k_run<POL, true, false> : (const void *)k_run<POL, false, false>;
+const void *run_fn(bool smem, bool ins, bool dense) {
+    if (ins) return smem ? (const void *)k_run<POL, true, true, false> : (const void *)k_run<POL, false, true, false>;
+    if (smem && dense) return (const void *)k_run<POL, true, false, true>;
+    return smem ? (const void *)k_run<POL, true, false, false> : (const void *)k_run<POL, false, false, false>;
 }
 
 template <int POL>
-void launch_pol(const RunParams &p, dim3 grid, dim3 block, size_t smem_bytes, cudaStream_t st) {
+void launch_pol(const RunParams &p, dim3 grid, dim3 block, size_t smem_bytes, bool dense, cudaStream_t st) {
     const bool sm = p.use_smem != 0;
     const bool ins = p.work_count != nullptr || p.batch_time != nullptr;
     if (ins) {
-        if (sm) k_run<POL, true, true><<<grid, block, smem_bytes, st>>>(p);
-        else k_run<POL, false, true><<<grid, block, smem_bytes, st>>>(p);
+        if (sm) k_run<POL, true, true, false><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, true, false><<<grid, block, smem_bytes, st>>>(p);
+    } else if (sm && dense) {
+        k_run<POL, true, false, true><<<grid, block, smem_bytes, st>>>(p);
     } else {
-        if (sm) k_run<POL, true, false><<<grid, block, smem_bytes, st>>>(p);
-        else k_run<POL, false, false><<<grid, block, smem_bytes, st>>>(p);
+        if (sm) k_run<POL, true, false, false><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, false, false><<<grid, block, smem_bytes, st>>>(p);
     }
 }
 
@@ -1618,27 +1624,28 @@ void launch_pol(const RunParams &p, dim3 grid, dim3 block, size_t smem_bytes, cu
 size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
-    for (int ins = 0; ins < 2; ++ins) {
-        const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true, ins)
-                         : policy == P_AMIN ? run_fn<P_AMIN>(true, ins)
-                         : policy == P_HSF  ? run_fn<P_HSF>(true, ins)
-                         : policy == P_AR   ? run_fn<P_AR>(true, ins)
-                                            : run_fn<P_AELL>(true, ins);
+    for (int v = 0; v < 3; ++v) {
+        const bool ins = v == 1, dense = v == 2;
+        const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true, ins, dense)
+                         : policy == P_AMIN ? run_fn<P_AMIN>(true, ins, dense)
+                         : policy == P_HSF  ? run_fn<P_HSF>(true, ins, dense)
+                         : policy == P_AR   ? run_fn<P_AR>(true, ins, dense)
+                                            : run_fn<P_AELL>(true, ins, dense);
         const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
 }
 
-cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes,
+cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes, bool dense,
                        cudaStream_t st) {
     const dim3 grid(blocks), block(32 * warps_per_block);
     switch (policy) {
-        case P_AMAX: launch_pol<P_AMAX>(p, grid, block, smem_bytes, st); break;
-        case P_AMIN: launch_pol<P_AMIN>(p, grid, block, smem_bytes, st); break;
-        case P_HSF: launch_pol<P_HSF>(p, grid, block, smem_bytes, st); break;
-        case P_AR: launch_pol<P_AR>(p, grid, block, smem_bytes, st); break;
-        default: launch_pol<P_AELL>(p, grid, block, smem_bytes, st); break;
+        case P_AMAX: launch_pol<P_AMAX>(p, grid, block, smem_bytes, dense, st); break;
+        case P_AMIN: launch_pol<P_AMIN>(p, grid, block, smem_bytes, dense, st); break;
+        case P_HSF: launch_pol<P_HSF>(p, grid, block, smem_bytes, dense, st); break;
+        case P_AR: launch_pol<P_AR>(p, grid, block, smem_bytes, dense, st); break;
+        default: launch_pol<P_AELL>(p, grid, block, smem_bytes, dense, st); break;
     }
     return cudaGetLastError();
 }

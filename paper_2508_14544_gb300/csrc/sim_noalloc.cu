@@ -172,7 +172,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.mainbuf = reinterpret_cast<simgb::QEnt *>(base + kOffMain);
     p.main_cap = kNaMaxPerInstance;
     const int blocks = int(std::min<int64_t>(kNaBlocks, (n_instances + kNaWarpsPerBlock - 1) / kNaWarpsPerBlock));
-    e = simgb::launch_run(policy, p, blocks, kNaWarpsPerBlock, 0, st);
+    e = simgb::launch_run(policy, p, blocks, kNaWarpsPerBlock, 0, false, st);
     if (e != cudaSuccess) return fail(SIM_E_CUDA, "sim_run_noalloc: simulation kernel launch failed");
     return SIM_OK;
 }

@@ -24,7 +24,8 @@ class Simulator:
                "warps_per_block": L.SIM_OPT_WARPS_PER_BLOCK, "smem_active_cap": L.SIM_OPT_SMEM_ACTIVE_CAP,
                "warps_per_sm": L.SIM_OPT_WARPS_PER_SM, "debug_checks": L.SIM_OPT_DEBUG_CHECKS,
                "tune_residency": L.SIM_OPT_TUNE_RESIDENCY, "evict_ties": L.SIM_OPT_EVICT_TIES,
-               "count_work": L.SIM_OPT_COUNT_WORK, "batch_time": L.SIM_OPT_BATCH_TIME}
+               "count_work": L.SIM_OPT_COUNT_WORK, "batch_time": L.SIM_OPT_BATCH_TIME,
+               "dense_residency": L.SIM_OPT_DENSE_RESIDENCY}
 
     def set_option(self, name: str, value: int) -> None:
         rc = L.sim_set_option(self.ctx, self.OPTIONS[name], int(value))
