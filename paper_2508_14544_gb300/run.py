@@ -2,6 +2,7 @@
 
   python -m paper_2508_14544_gb300.run --workload c2 --policy A_min [--instances 0:1024[:step]] [--repeat 1]
                                        [--warps-per-block W] [--warps-per-sm S] [--evict-ties-by-index]
+                                       [--dense]
 
 Prints one JSON line per run with the wall time of sim_run, totals of the result fields, the
 throughput and a sha256 of the per-instance result records (equal across runs and launch shapes).
@@ -28,6 +29,7 @@ def main(argv=None) -> None:
     ap.add_argument("--warps-per-block", type=int, default=0)
     ap.add_argument("--warps-per-sm", type=int, default=0, help="residency limit (4: one warp per scheduler)")
     ap.add_argument("--evict-ties-by-index", action="store_true", help="A_min: cancellation ties by index")
+    ap.add_argument("--dense", action="store_true", help="12 simulating warps per SM, 384 active-set slots")
     args = ap.parse_args(argv)
     ids = None
     if args.instances:
@@ -43,6 +45,8 @@ def main(argv=None) -> None:
         opts["warps_per_sm"] = args.warps_per_sm
     if args.evict_ties_by_index:
         opts["evict_ties"] = 1
+    if args.dense:
+        opts["dense_residency"] = 1
     with Simulator(POLICIES[args.policy], w.M, w.n_instances, **opts) as sim:
         sim.set_tie_seeds(w.tie_seeds())
         for _ in range(args.repeat):
