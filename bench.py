@@ -370,22 +370,43 @@ def run_ours(args) -> None:
         total_s = float(t.item())
     value = rs_per_step * args.steps * world / total_s
 
-    # end to end through the public API with host (pinned) buffers: H2D inside sim_load, D2H of
-    # the per-instance results inside sim_run and of the ratios
-    e2e_steps = max(1, min(args.steps, 3))
-    host_in = [p.numpy() for p in pinned]
-    torch.cuda.synchronize()
+    # end to end through the public API from pinned host buffers: every step copies its inputs
+    # (the five request arrays, shared by the three policies) host to device on a copy stream and
+    # reads every policy's per-instance results and the ratios back.  The device inputs are double
+    # buffered, so step k+1's copy runs while step k simulates; step 0's copy is not hidden.  One
+    # untimed pass first (the first transfers from a pinned buffer are slower than the rest).
+    e2e_steps = args.steps
+    copy_stream = torch.cuda.Stream(device=dev)
+    bufs = [[torch.empty_like(t) for t in d_in] for _ in range(2)]
+    copied = [torch.cuda.Event() for _ in range(2)]
+
+    def copy_in(k):
+        with torch.cuda.stream(copy_stream):
+            for dst, src in zip(bufs[k % 2], pinned):
+                dst.copy_(src, non_blocking=True)
+            copied[k % 2].record(copy_stream)
+
+    def e2e_run(n_steps):
+        copy_in(0)
+        for k in range(n_steps):
+            copied[k % 2].synchronize()
+            if k + 1 < n_steps:
+                copy_in(k + 1)  # the other buffer: its last reader, step k-1's staging, has finished
+            step(bufs[k % 2])
+        torch.cuda.synchronize()
+
+    e2e_run(1)
+    if world > 1:
+        dist.barrier()
     t0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        step(host_in)
-    torch.cuda.synchronize()
+    e2e_run(e2e_steps)
     e2e_s = time.perf_counter() - t0
     if world > 1:
         t = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
     e2e_val = rs_per_step * e2e_steps * world / e2e_s
-    h2d = 3 * 5 * w.n_total * 4
+    h2d = 5 * w.n_total * 4
     d2h = 3 * w.n_instances * 56 + 2 * w.n_instances * 8
 
     if rank != 0:
