@@ -337,7 +337,7 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     dense = dense && smem && !c->count_work && !c->batch_time;
     int wpb = dense ? simgb::kDenseWarps : c->wpb;
-    const int dcap = c->dcap;
+    const int dcap = dense ? simgb::kDenseDcap : c->dcap;
     int ca = smem ? (dense ? simgb::kDenseCa : c->smem_ca) : ((std::max(c->n_max, 128) + 127) / 128) * 128;
     size_t per_warp = simgb::warp_ws_bytes(ca, dcap);
     size_t smem_bytes = 0;

@@ -95,6 +95,7 @@ cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per
                        cudaStream_t st);
 constexpr int kDenseCa = 384;      // active-set slots per warp of the dense configuration
 constexpr int kDenseWarps = 4;     // warps per block of the dense configuration
+constexpr int kDenseDcap = 256;    // delta-queue capacity per warp of the dense configuration
 cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
 cudaError_t launch_batch_time(const int64_t *sums, const DevResult *res, const double *coef, double *out, int32_t n,
                               cudaStream_t st);

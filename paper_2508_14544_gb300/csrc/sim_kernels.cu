@@ -1062,7 +1062,8 @@ __device__ __forceinline__ void sort_admitted(const Ws &w, int K, QEnt &mine) {
 }
 
 // First step tau in (t, tau_lim) at which the head candidate (prompt s, estimate L) fits, with the
-// active set unchanged; kBig if none.  In terms of y = tau + L - 1, the interval between active
+// active set unchanged; kBig if none; -1 if the answer needs the arrays and arrays_ok is false
+// (they hold cancelled jobs whose compaction was deferred).  In terms of y = tau + L - 1, the interval between active
 // endpoints (E[j-1], E[j]] has #{E < y} = j, and #{E <= y} = j below E[j] and the end of E[j]'s
 // group at y = E[j] (whose prefix maximum is PM[j+1]: within a group of equal E that lies at or
 // after tb the first entry has the largest H).  Conditions (1)-(3) give, per interval, a lower
@@ -1071,7 +1072,7 @@ __device__ __forceinline__ void sort_admitted(const Ws &w, int K, QEnt &mine) {
 // shared-memory kernel); PM[0] is the -infinity sentinel and takes no arithmetic.
 template <bool N>
 __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, int SB0, int64_t M, int t, int s,
-                                                  int L, int64_t tau_lim) {
+                                                  int L, int64_t tau_lim, bool arrays_ok) {
     using W = wint<N>;
     const int lane = lane_id();
     const W BIG = N ? W(1 << 29) : W(int64_t(1) << 60);
@@ -1080,6 +1081,7 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
     const W tau1 = floor_div32(M - s - 1 - SB0, A);  // (1)
     const W yup = min(ylim, tau1 + L - 1);
     if (yup <= y0) return kBig;
+    if (!arrays_ok) return -1;  // the arrays hold cancelled jobs: the caller compacts them first
     const W C = W(M) - s - L;  // (2): PM - C <= y;  (3): y <= floor((C - SB[j]) / (A - j))
     W best = BIG;
     #pragma unroll 1
@@ -1193,7 +1195,10 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     // (steps and request steps have their own counters).
     const bool bt = INS && P.batch_time != nullptr;
     int64_t bx0 = 0, bx1 = 0, bx2 = 0, bx3 = 0, bmem = 0, bpf = 0;
-    int A = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
+    // A: live jobs; Ad: entries of the active-set arrays, which after an A_min cancellation whose
+    // compaction is deferred also hold the cancelled jobs (F = -1).  SB0 and A are exact either way;
+    // SB and PM describe the arrays only when Ad == A.
+    int A = 0, Ad = 0, tb = 0, SB0 = 0, nextF = INT_MAX;
     if (lane == 0) {  // derived arrays of the empty active set (the workspace is reused)
         w.SB[0] = 0;
         w.PM[0] = INT_MIN;
@@ -1223,7 +1228,8 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             // instruction cache.
             tb = tb_next;
             const int A0 = A;
-            compact_derive<N>(w, A, tb, SB0, nextF);
+            compact_derive<N>(w, Ad, tb, SB0, nextF);
+            A = Ad;
             pend_compact = false;
             pdirty = true;
             if (done_step) {  // the jobs completed at step tb - 1 (C = tb) have left the set
@@ -1295,19 +1301,20 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 // One-chunk sets keep the lane's four estimates in registers for all of the step's
                 // cancellations, `live` marking those still in the set (the array itself is never
                 // written by a run-time position, which would put it in local memory).
-                const bool reg = A <= kChunk;
+                const bool reg = Ad <= kChunk;
                 unsigned rk[4] = {0u, 0u, 0u, 0u};
                 unsigned live = 0;
                 if (reg) {
                     const int base = 4 * lane;
-                    const int4 k4 = ld4(w.K, base);
-                    const int kk[4] = {k4.x, k4.y, k4.z, k4.w};
+                    const int4 k4 = ld4(w.K, base), f4 = ld4(w.F, base);
+                    const int kk[4] = {k4.x, k4.y, k4.z, k4.w}, ff[4] = {f4.x, f4.y, f4.z, f4.w};
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         rk[j] = unsigned(kk[j]);
-                        if (base + j < A) live |= 1u << j;
+                        if (base + j < Ad && ff[j] >= 0) live |= 1u << j;
                     }
                 }
+                bool defer = !P.debug;  // no cancelled job is the next to complete
                 #pragma unroll 1
                 while (need > wint<N>(M)) {
                     int pos = -1;
@@ -1328,13 +1335,13 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                         unsigned bk = UINT_MAX;
                         int bc = 0, bp = -1;
                         #pragma unroll 1
-                        for (int cb = 0; cb < A; cb += kChunk) {
+                        for (int cb = 0; cb < Ad; cb += kChunk) {
                             const int base = cb + 4 * lane;
                             const int4 f4 = ld4(w.F, base), k4 = ld4(w.K, base);
                             const int ff[4] = {f4.x, f4.y, f4.z, f4.w}, kk[4] = {k4.x, k4.y, k4.z, k4.w};
 #pragma unroll
                             for (int j = 0; j < 4; ++j) {
-                                if (base + j < A && ff[j] >= 0) {
+                                if (base + j < Ad && ff[j] >= 0) {
                                     const unsigned k = unsigned(kk[j]);
                                     if (k < bk) {
                                         bk = k;
@@ -1352,7 +1359,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                         if (b) pos = __shfl_sync(FULL, bp, __ffs(b) - 1);
                     }
                     if (mk == UINT_MAX) pos = -1;
-                    else if (tot > 1) pos = tie_position(w.F, w.K, w.I, A, mk, tie_base(tie_seed, t), P.evict_index == 0);
+                    else if (tot > 1) pos = tie_position(w.F, w.K, w.I, Ad, mk, tie_base(tie_seed, t), P.evict_index == 0);
                     if (reg && pos >= 0 && (pos >> 2) == lane) live &= ~(1u << (pos & 3));
                     if (pos < 0) {  // UINT_MAX: no live entry
                         status = ST_STATE;
@@ -1368,14 +1375,25 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     if (lane == 0) w.F[pos] = -1;
                     __syncwarp();
                     need -= wint<N>(b) + t;
+                    SB0 -= b + tb;
+                    --A;
+                    if (f == nextF) defer = false;
                     ++nev;
                     if (INS) ++ev_step;
                     delta_insert(w, q, e, gbp);
                 }
                 if (status != ST_OK) break;
-                tb_next = t;
-                pend_compact = true;
+                // The cancelled jobs stay in the arrays (F = -1) until the next compaction, which
+                // happens when something reads SB, PM or the order of the arrays (an admission
+                // test past its O(1) part, a first-fit search, an insertion) or after the next
+                // completion step; until then SB0, A and nextF describe the live jobs.  On the
+                // 40960 x 2000 workload 62 % of the steps with cancellations need no compaction
+                // of their own.
                 hvalid = false;
+                if (!defer) {
+                    tb_next = t;
+                    pend_compact = true;
+                }
                 continue;
             }
         }
@@ -1419,6 +1437,11 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             const wint<N> dt = wint<N>(t) - tb;
             const wint<N> need = wint<N>(SB0) + wint<N>(A) * dt;
             bool fits = need + h.s + 1 <= wint<N>(M);
+            if (fits && Ad > A) {  // the rest of the test reads the arrays: compact them first
+                tb_next = tb;
+                pend_compact = true;
+                break;
+            }
             if (fits && A > 0) {
                 const int64_t y = int64_t(t) + h.key - 1;
                 if (pdirty || y != y_prev + 1) {
@@ -1466,6 +1489,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 status = kStatusCapacity;
                 break;
             }
+            Ad = A;
             tb = t;
             if (A <= kChunk) derive_one<N>(w, A, tb, SB0, nextF);
             else derive<N>(w, A, tb, SB0, nextF);
@@ -1482,6 +1506,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             hvalid = false;
         }
         if (status != ST_OK) break;
+        if (pend_compact) continue;  // the admission test asked for the deferred compaction
         // ---- S6: process the batch
         if (t == nextF) {
             const wint<N> mem = wint<N>(SB0) + wint<N>(A) * (wint<N>(t) - tb);
@@ -1503,7 +1528,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             // iteration removes them (F < the new time base) and counts them
             if (P.completion) {
 #pragma unroll 1
-                for (int i = lane; i < A; i += 32)
+                for (int i = lane; i < Ad; i += 32)
                     if (w.F[i] == t) P.completion[info.base + w.I[i]] = int64_t(t) + 1;
             }
             makespan = int64_t(t) + 1;
@@ -1520,8 +1545,15 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             if (POL == P_AELL && A > 0) tau = min(tau, int64_t(w.E[0]) + 1);
             tau = min(tau, int64_t(t) + (cap - steps));
             tau = min(tau, int64_t(kMaxStep) + 1);
-            if (tau > int64_t(t) + 1 && hvalid && A > 0)
-                tau = min(tau, first_fit_step<N>(w, A, tb, SB0, M, t, h.s, h.key, tau));
+            if (tau > int64_t(t) + 1 && hvalid && A > 0) {
+                const int64_t ff = first_fit_step<N>(w, A, tb, SB0, M, t, h.s, h.key, tau, Ad == A);
+                if (ff < 0) {  // the search reads the arrays: compact them first
+                    tb_next = tb;
+                    pend_compact = true;
+                    continue;
+                }
+                tau = min(tau, ff);
+            }
             const int64_t c = max(tau - int64_t(t), int64_t(1));
             const int64_t mem = int64_t(SB0) + int64_t(A) * (int64_t(t) + c - 1 - tb);
             if (mem > M) {
@@ -1573,18 +1605,22 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
 }
 
 // DENSE: the copy for three blocks of four warps per SM (12 simulating warps, at most 170
-// registers a thread), which the host pairs with a 384-slot shared-memory active set; otherwise
-// blocks of up to 256 threads and as many registers as the code wants (two blocks per SM).
+// registers a thread), with the workspace layout fixed at compile time (384 active-set slots, a
+// 256-entry delta): the workspace arrays are then constant offsets from one shared-memory base
+// instead of pointers held in registers.  Otherwise blocks of up to 256 threads, as many
+// registers as the code wants (two blocks per SM) and the layout of P.ca and P.dcap.
 template <int POL, bool SMEM, bool INS, bool DENSE>
 __global__ void __launch_bounds__(DENSE ? 128 : 256, DENSE ? 3 : 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
     const int wib = threadIdx.x >> 5;
     const int64_t slot = int64_t(blockIdx.x) * (blockDim.x >> 5) + wib;
+    const int ca = DENSE ? kDenseCa : P.ca;
+    const int dcap = DENSE ? kDenseDcap : P.dcap;
     unsigned char *base;
-    if (SMEM) base = smem_raw + size_t(wib) * ws_bytes_impl(P.ca, P.dcap);
+    if (SMEM) base = smem_raw + size_t(wib) * ws_bytes_impl(ca, dcap);
     else base = P.gws + slot * P.gws_stride;
-    Ws w = carve_ws(base, P.ca, P.dcap);
+    Ws w = carve_ws(base, ca, dcap);
     w.mb0 = P.mainbuf + slot * 2 * P.main_cap;
     w.mb1 = w.mb0 + P.main_cap;
     for (;;) {
