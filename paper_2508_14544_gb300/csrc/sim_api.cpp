@@ -40,8 +40,7 @@ struct sim_ctx {
     int tuned_wps = 0;
     int tuned_dense = 0;
     int64_t tuned_shape[3] = {-1, -1, -1};
-    int smem_ca = 512;
-    int dcap = 256;
+    int smem_ca = simgb::kSmemCaDefault;
     // state
     int device = -1;
     bool loaded = false;
@@ -337,9 +336,8 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     dense = dense && smem && !c->count_work && !c->batch_time;
     int wpb = dense ? simgb::kDenseWarps : c->wpb;
-    const int dcap = dense ? simgb::kDenseDcap : c->dcap;
     int ca = smem ? (dense ? simgb::kDenseCa : c->smem_ca) : ((std::max(c->n_max, 128) + 127) / 128) * 128;
-    size_t per_warp = simgb::warp_ws_bytes(ca, dcap);
+    size_t per_warp = simgb::warp_ws_bytes(ca);
     size_t smem_bytes = 0;
     if (smem) {
         while (wpb > 1 && per_warp * wpb > size_t(smem_optin)) --wpb;
@@ -396,7 +394,6 @@ static int run_launch(sim_ctx *c, cudaStream_t st, const int32_t *work_dev, int3
     p.work_count = c->count_work ? c->d_wc : nullptr;
     p.batch_time = c->batch_time ? c->d_bt : nullptr;
     p.ca = ca;
-    p.dcap = dcap;
     p.use_smem = smem ? 1 : 0;
     p.debug = c->debug_checks;
     p.evict_index = c->evict_index;

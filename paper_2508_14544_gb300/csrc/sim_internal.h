@@ -77,7 +77,6 @@ struct RunParams {
     int64_t *batch_time;       // optional, 6 per instance: the batch-time sums X0..X3, F2, F3
     // workspace
     int32_t ca;                // active-set capacity per instance (multiple of 32)
-    int32_t dcap;              // delta-queue capacity per instance (multiple of 32)
     int32_t use_smem;          // 1: active set + delta queue in shared memory; 0: global workspace
     int32_t debug;             // 1: check the simulation state's invariants every iteration (global kernel)
     int32_t evict_index;       // 1: A_min eviction ties by request index instead of the random tie key
@@ -87,15 +86,16 @@ struct RunParams {
     int64_t main_cap;
 };
 
-size_t warp_ws_bytes(int ca, int dcap);
+size_t warp_ws_bytes(int ca);  // workspace bytes per warp slot for ca active-set slots
 
 cudaError_t launch_stage(const StageParams &p, cudaStream_t st);
-// dense: the 12-warps-per-SM copy of the plain shared-memory kernel (blocks of 4 warps)
+// dense: the 12-warps-per-SM copy of the plain shared-memory kernel (blocks of 4 warps, kDenseCa slots)
 cudaError_t launch_run(int policy, const RunParams &p, int blocks, int warps_per_block, size_t smem_bytes, bool dense,
                        cudaStream_t st);
 constexpr int kDenseCa = 384;      // active-set slots per warp of the dense configuration
 constexpr int kDenseWarps = 4;     // warps per block of the dense configuration
-constexpr int kDenseDcap = 256;    // delta-queue capacity per warp of the dense configuration
+constexpr int kSmemCaDefault = 512;  // active-set slots per warp in shared memory by default
+constexpr int kDcap = 256;         // delta-queue capacity per warp slot (multiple of 32)
 cudaError_t launch_ratio(const DevResult *pol, const DevResult *ref, double *out, int32_t n, cudaStream_t st);
 cudaError_t launch_batch_time(const int64_t *sums, const DevResult *res, const double *coef, double *out, int32_t n,
                               cudaStream_t st);

@@ -1604,23 +1604,23 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     __syncwarp();
 }
 
-// DENSE: the copy for three blocks of four warps per SM (12 simulating warps, at most 170
-// registers a thread), with the workspace layout fixed at compile time (384 active-set slots, a
-// 256-entry delta): the workspace arrays are then constant offsets from one shared-memory base
-// instead of pointers held in registers.  Otherwise blocks of up to 256 threads, as many
-// registers as the code wants (two blocks per SM) and the layout of P.ca and P.dcap.
-template <int POL, bool SMEM, bool INS, bool DENSE>
-__global__ void __launch_bounds__(DENSE ? 128 : 256, DENSE ? 3 : 1) k_run(RunParams P) {
+// LAY: the workspace layout.  1 (dense): three blocks of four warps per SM (12 simulating warps,
+// at most 170 registers a thread) and kDenseCa active-set slots; 2: the default kSmemCaDefault
+// slots; 0: P.ca slots (the global-memory kernel, other shared-memory capacities and the
+// instrumented copy).  With 1 and 2 the layout is fixed at compile time, so the workspace arrays
+// are constant offsets from one shared-memory base instead of pointers held in registers.  Other
+// than dense: blocks of up to 256 threads and as many registers as the code wants.
+template <int POL, bool SMEM, bool INS, int LAY>
+__global__ void __launch_bounds__(LAY == 1 ? 128 : 256, LAY == 1 ? 3 : 1) k_run(RunParams P) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int lane = lane_id();
     const int wib = threadIdx.x >> 5;
     const int64_t slot = int64_t(blockIdx.x) * (blockDim.x >> 5) + wib;
-    const int ca = DENSE ? kDenseCa : P.ca;
-    const int dcap = DENSE ? kDenseDcap : P.dcap;
+    const int ca = LAY == 1 ? kDenseCa : (LAY == 2 ? kSmemCaDefault : P.ca);
     unsigned char *base;
-    if (SMEM) base = smem_raw + size_t(wib) * ws_bytes_impl(ca, dcap);
+    if (SMEM) base = smem_raw + size_t(wib) * ws_bytes_impl(ca, kDcap);
     else base = P.gws + slot * P.gws_stride;
-    Ws w = carve_ws(base, ca, dcap);
+    Ws w = carve_ws(base, ca, kDcap);
     w.mb0 = P.mainbuf + slot * 2 * P.main_cap;
     w.mb1 = w.mb0 + P.main_cap;
     for (;;) {
@@ -1633,11 +1633,16 @@ __global__ void __launch_bounds__(DENSE ? 128 : 256, DENSE ? 3 : 1) k_run(RunPar
     }
 }
 
+// The shared-memory copies: v = 0 plain with P.ca slots, 1 instrumented, 2 dense, 3 plain with
+// the default slots.
 template <int POL>
-const void *run_fn(bool smem, bool ins, bool dense) {
-    if (ins) return smem ? (const void *)k_run<POL, true, true, false> : (const void *)k_run<POL, false, true, false>;
-    if (smem && dense) return (const void *)k_run<POL, true, false, true>;
-    return smem ? (const void *)k_run<POL, true, false, false> : (const void *)k_run<POL, false, false, false>;
+const void *smem_fn(int v) {
+    switch (v) {
+        case 0: return (const void *)k_run<POL, true, false, 0>;
+        case 1: return (const void *)k_run<POL, true, true, 0>;
+        case 2: return (const void *)k_run<POL, true, false, 1>;
+        default: return (const void *)k_run<POL, true, false, 2>;
+    }
 }
 
 template <int POL>
@@ -1645,28 +1650,29 @@ void launch_pol(const RunParams &p, dim3 grid, dim3 block, size_t smem_bytes, bo
     const bool sm = p.use_smem != 0;
     const bool ins = p.work_count != nullptr || p.batch_time != nullptr;
     if (ins) {
-        if (sm) k_run<POL, true, true, false><<<grid, block, smem_bytes, st>>>(p);
-        else k_run<POL, false, true, false><<<grid, block, smem_bytes, st>>>(p);
+        if (sm) k_run<POL, true, true, 0><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, true, 0><<<grid, block, smem_bytes, st>>>(p);
     } else if (sm && dense) {
-        k_run<POL, true, false, true><<<grid, block, smem_bytes, st>>>(p);
+        k_run<POL, true, false, 1><<<grid, block, smem_bytes, st>>>(p);
+    } else if (sm && p.ca == kSmemCaDefault) {
+        k_run<POL, true, false, 2><<<grid, block, smem_bytes, st>>>(p);
     } else {
-        if (sm) k_run<POL, true, false, false><<<grid, block, smem_bytes, st>>>(p);
-        else k_run<POL, false, false, false><<<grid, block, smem_bytes, st>>>(p);
+        if (sm) k_run<POL, true, false, 0><<<grid, block, smem_bytes, st>>>(p);
+        else k_run<POL, false, false, 0><<<grid, block, smem_bytes, st>>>(p);
     }
 }
 
 }  // namespace
 
-size_t warp_ws_bytes(int ca, int dcap) { return ws_bytes_impl(ca, dcap); }
+size_t warp_ws_bytes(int ca) { return ws_bytes_impl(ca, kDcap); }
 
 cudaError_t set_run_smem_limit(int policy, size_t bytes) {
-    for (int v = 0; v < 3; ++v) {
-        const bool ins = v == 1, dense = v == 2;
-        const void *fn = policy == P_AMAX ? run_fn<P_AMAX>(true, ins, dense)
-                         : policy == P_AMIN ? run_fn<P_AMIN>(true, ins, dense)
-                         : policy == P_HSF  ? run_fn<P_HSF>(true, ins, dense)
-                         : policy == P_AR   ? run_fn<P_AR>(true, ins, dense)
-                                            : run_fn<P_AELL>(true, ins, dense);
+    for (int v = 0; v < 4; ++v) {
+        const void *fn = policy == P_AMAX ? smem_fn<P_AMAX>(v)
+                         : policy == P_AMIN ? smem_fn<P_AMIN>(v)
+                         : policy == P_HSF  ? smem_fn<P_HSF>(v)
+                         : policy == P_AR   ? smem_fn<P_AR>(v)
+                                            : smem_fn<P_AELL>(v);
         const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
         if (e != cudaSuccess) return e;
     }

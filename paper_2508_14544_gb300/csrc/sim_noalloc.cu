@@ -36,7 +36,7 @@ constexpr int64_t kNaMaxPerInstance = 2048;       // requests per instance
 constexpr int kNaWarpsPerBlock = 4;
 constexpr int kNaBlocks = 32;
 constexpr int64_t kNaSlots = int64_t(kNaBlocks) * kNaWarpsPerBlock;  // simulating warps
-constexpr int kNaDeltaCap = 256;
+constexpr int kNaDeltaCap = simgb::kDcap;
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -97,7 +97,7 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     if (nt > 0 && (!arrival_t || !prompt_s || !lower_l || !upper_u || !true_o))
         return fail(SIM_E_INVAL, "sim_run_noalloc: NULL input array");
 
-    if (simgb::warp_ws_bytes(int(kNaMaxPerInstance), kNaDeltaCap) > ws_bytes_max())
+    if (simgb::warp_ws_bytes(int(kNaMaxPerInstance)) > ws_bytes_max())
         return fail(SIM_E_STATE, "sim_run_noalloc: workspace layout mismatch");
     int dev = -1;
     cudaError_t e = cudaGetDevice(&dev);
@@ -163,7 +163,6 @@ extern "C" int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const
     p.work_count = nullptr;
     p.batch_time = nullptr;
     p.ca = int32_t(((std::max<int64_t>(n_max, 128) + 127) / 128) * 128);  // >= any active set: no fallback
-    p.dcap = kNaDeltaCap;
     p.use_smem = 0;
     p.debug = 0;
     p.evict_index = 0;
