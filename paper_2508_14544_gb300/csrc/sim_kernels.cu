@@ -1078,6 +1078,8 @@ __device__ __forceinline__ int64_t first_fit_step(const Ws &w, int A, int tb, in
     const W BIG = N ? W(1 << 29) : W(int64_t(1) << 60);
     const W y0 = W(t - tb) + L - 1;
     const W ylim = W(min(tau_lim - tb, int64_t(BIG))) - 1 + L - 1;
+    // (1) already fails at step t + 1 (the usual case, tested without the division below)
+    if (int64_t(SB0) + int64_t(A) * (int64_t(t) + 1 - tb) + s + 1 > M) return kBig;
     const W tau1 = floor_div32(M - s - 1 - SB0, A);  // (1)
     const W yup = min(ylim, tau1 + L - 1);
     if (yup <= y0) return kBig;
@@ -1381,6 +1383,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     ++nev;
                     if (INS) ++ev_step;
                     delta_insert(w, q, e, gbp);
+                    if (hvalid && qless(e, h)) h = e;  // the head of R_t is the smaller of the two
                 }
                 if (status != ST_OK) break;
                 // The cancelled jobs stay in the arrays (F = -1) until the next compaction, which
@@ -1389,7 +1392,6 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 // completion step; until then SB0, A and nextF describe the live jobs.  On the
                 // 40960 x 2000 workload 62 % of the steps with cancellations need no compaction
                 // of their own.
-                hvalid = false;
                 if (!defer) {
                     tb_next = t;
                     pend_compact = true;
