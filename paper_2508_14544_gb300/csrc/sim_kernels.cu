@@ -1209,15 +1209,17 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
     int t = ra[0];
     int ap = 0;
     int next_a = t;
-    int64_t sumC = 0, peak = 0, steps = 0, rsteps = 0, nev = 0;
-    int64_t makespan = 0;
+    int64_t sumC = 0, rsteps = 0, nev = 0;
+    // 32 bits suffice (fewer live registers): steps <= t + 1 and makespan <= t + 1 with
+    // t <= kMaxStep + 1, and the peak is a step's memory, <= M <= 2^26
+    int steps = 0, makespan = 0, peak = 0;
     int ndone = 0;
     int status = ST_OK;
 
     bool hvalid = false;
     QEnt h;
     bool pdirty = true;
-    int64_t y_prev = 0;
+    int y_prev = 0;  // t + key - 1 <= kMaxStep + 2^26 < 2^31
     int hi = 0, lb = 0;
 
     bool pend_compact = false, done_step = false;
@@ -1446,7 +1448,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
             }
             if (fits && A > 0) {
                 const int64_t y = int64_t(t) + h.key - 1;
-                if (pdirty || y != y_prev + 1) {
+                if (pdirty || y != int64_t(y_prev) + 1) {
                     prefix_le_lt(w.E, A, y, hi, lb);
                 } else {
                     lb = hi;
@@ -1454,7 +1456,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                     while (hi < A && w.E[hi] <= y) ++hi;
                 }
                 pdirty = false;
-                y_prev = y;
+                y_prev = int(y);
                 // PM[0] is the INT_MIN sentinel: compare without adding to it
                 if (wint<N>(w.PM[hi]) > wint<N>(M) - h.s - 1 + dt) fits = false;
                 const wint<N> v = wint<N>(w.SB[lb]) + wint<N>(A - lb) * wint<N>(y - tb);
@@ -1516,7 +1518,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 status = ST_STATE;
                 break;
             }
-            if (mem > peak) peak = mem;
+            if (mem > peak) peak = int(mem);
             rsteps += A;
             ++steps;
             if (bt) bmem += int64_t(mem);
@@ -1533,7 +1535,7 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 for (int i = lane; i < Ad; i += 32)
                     if (w.F[i] == t) P.completion[info.base + w.I[i]] = int64_t(t) + 1;
             }
-            makespan = int64_t(t) + 1;
+            makespan = t + 1;
             tb_next = t + 1;
             pend_compact = true;
             done_step = true;
@@ -1562,9 +1564,9 @@ __device__ __forceinline__ void sim_instance(const RunParams &P, const Ws &w0, i
                 status = ST_STATE;
                 break;
             }
-            if (mem > peak) peak = mem;
+            if (mem > peak) peak = int(mem);
             rsteps += int64_t(A) * c;
-            steps += c;
+            steps += int(c);
             if (bt)  // steps t .. t+c-1 have memory SB0 + A (x - tb)
                 bmem += c * int64_t(SB0) + int64_t(A) * (c * (int64_t(t) - tb) + c * (c - 1) / 2);
             if (INS) {
