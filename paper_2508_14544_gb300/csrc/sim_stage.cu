@@ -56,9 +56,9 @@ __device__ void bitonic_sort(QEnt *R, int32_t *RA, int n) {
     int N = 1;
     while (N < n) N <<= 1;
     for (int k = 2; k <= N; k <<= 1) {
-        for (int d = k >> 1; d >= 1; d >>= 1) {
+        for (int d = k >> 1, ld = __ffs(d) - 1; d >= 1; d >>= 1, --ld) {
             for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
-                const int i = (p / d) * 2 * d + (p % d);
+                const int i = ((p >> ld) << (ld + 1)) | (p & (d - 1));  // d is a power of two
                 const int j = (d == (k >> 1)) ? (i | (k - 1)) - (i & (k - 1)) : i + d;  // first pass: mirror
                 if (j < n) {
                     const QEnt x = R[i], y = R[j];
@@ -76,39 +76,103 @@ __device__ void bitonic_sort(QEnt *R, int32_t *RA, int n) {
     }
 }
 
-// The same order for an instance held in shared memory as 12-byte pairs: the key (a << 32 | policy
-// key; both are >= 0 in a valid instance, so the unsigned order is the (a, key) order) and the
-// request index; the prompt and true lengths stay in place, indexed by request.
-__device__ __forceinline__ void bitonic_sort_pairs(uint64_t *sk, int32_t *si, int n) {
-    int N = 1;
-    while (N < n) N <<= 1;
-    for (int k = 2; k <= N; k <<= 1) {
-        for (int d = k >> 1; d >= 1; d >>= 1) {
-            for (int p = threadIdx.x; p < N / 2; p += blockDim.x) {
-                const int i = (p / d) * 2 * d + (p % d);
-                const int j = (d == (k >> 1)) ? (i | (k - 1)) - (i & (k - 1)) : i + d;
-                if (j < n) {
-                    const uint64_t ki = sk[i], kj = sk[j];
-                    const int ii = si[i], ij = si[j];
-                    if (kj < ki || (kj == ki && ij < ii)) {
-                        sk[i] = kj;
-                        sk[j] = ki;
-                        si[i] = ij;
-                        si[j] = ii;
-                    }
-                }
-            }
-            __syncthreads();
-        }
+// Instances of up to this many requests are sorted in shared memory: per request its key, arrival,
+// prompt and true length and two index buffers (24 bytes), plus the radix counters.
+constexpr int kStageSmemN = 2048;
+constexpr int kStageSmemBytesPerReq = 24;
+constexpr int kStageSmemIpt = kStageSmemN / 256;  // elements per thread of a radix pass
+constexpr size_t kStageCntBytes = size_t(16) * kStageSmemIpt * 8 * sizeof(uint16_t);
+
+// Instances held in shared memory are sorted by an LSD radix sort of request indices, 4-bit digits
+// of the policy key and then of the arrival step, each pass stable, so the order is (a, key, idx)
+// (both are >= 0 in a valid instance).  A pass ranks element e = r * 256 + thread (iteration r):
+// within a warp and iteration, __match_any_sync groups the lanes with equal digits and a lane's
+// rank in its group is the number of group lanes below it; the groups' sizes go to counters in
+// (digit, iteration, warp) order, whose exclusive prefix sums are the groups' first output
+// positions.  Elements are thereby placed in (digit, e) order: stable.
+constexpr int kRadixBits = 4;
+constexpr int kRadixBins = 1 << kRadixBits;
+constexpr int kStageThreads = 256;
+constexpr int kStageWarps = kStageThreads / 32;
+
+template <int IPT>
+__device__ __forceinline__ void radix_pass(const int32_t *keyof, const int32_t *in, int32_t *out, uint16_t *cnt,
+                                           int *wsum, int n, int shift) {
+    constexpr int kCnt = kRadixBins * IPT * kStageWarps;  // a multiple of 4 * kStageThreads / 4
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const unsigned lt = (1u << lane) - 1u;
+    for (int f = t; f < kCnt; f += kStageThreads) cnt[f] = 0;
+    __syncthreads();
+    int dg[IPT], rk[IPT], ix[IPT];
+#pragma unroll
+    for (int r = 0; r < IPT; ++r) {
+        const int e = r * kStageThreads + t;
+        const bool v = e < n;
+        ix[r] = v ? in[e] : 0;
+        dg[r] = v ? ((keyof[ix[r]] >> shift) & (kRadixBins - 1)) : kRadixBins;  // past the end: a group of its own
+        const unsigned peers = __match_any_sync(FULL, dg[r]);
+        rk[r] = __popc(peers & lt);
+        if (v && rk[r] == 0) cnt[(dg[r] * IPT + r) * kStageWarps + w] = uint16_t(__popc(peers));
     }
+    __syncthreads();
+    // exclusive prefix sums of the counters, kCnt / kStageThreads consecutive ones per thread
+    constexpr int kPer = kCnt / kStageThreads;
+    int c[kPer], sum = 0;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        c[i] = cnt[kPer * t + i];
+        sum += c[i];
+    }
+    int x = sum;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_up_sync(FULL, x, d);
+        if (lane >= d) x += y;
+    }
+    if (lane == 31) wsum[w] = x;
+    __syncthreads();
+    int run = x - sum;
+    for (int i = 0; i < w; ++i) run += wsum[i];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        cnt[kPer * t + i] = uint16_t(run);
+        run += c[i];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < IPT; ++r) {
+        const int e = r * kStageThreads + t;
+        if (e < n) out[cnt[(dg[r] * IPT + r) * kStageWarps + w] + rk[r]] = ix[r];
+    }
+    __syncthreads();
 }
 
-// Instances of up to this many requests are sorted in shared memory (20 bytes per request).
-constexpr int kStageSmemN = 2048;
-constexpr int kStageSmemBytesPerReq = 20;
+// Sorts the indices 0..n-1 held in i0 (scratch i1) by (ka, kk, index); returns the buffer that
+// holds the result.  kmax, amax: the largest key and arrival step (>= 0).
+__device__ int32_t *radix_sort_idx(const int32_t *kk, const int32_t *ka, int32_t *i0, int32_t *i1, uint16_t *cnt,
+                                   int *wsum, int n, int kmax, int amax) {
+    int32_t *in = i0, *out = i1;
+    const int kbits = kmax > 0 ? 32 - __clz(kmax) : 0;
+    const int abits = amax > 0 ? 32 - __clz(amax) : 0;
+    for (int sh = 0; sh < kbits; sh += kRadixBits) {
+        radix_pass<kStageSmemIpt>(kk, in, out, cnt, wsum, n, sh);
+        int32_t *tmp = in;
+        in = out;
+        out = tmp;
+    }
+    for (int sh = 0; sh < abits; sh += kRadixBits) {
+        radix_pass<kStageSmemIpt>(ka, in, out, cnt, wsum, n, sh);
+        int32_t *tmp = in;
+        in = out;
+        out = tmp;
+    }
+    return in;
+}
 
-__global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
+
+__global__ void __launch_bounds__(kStageThreads) k_stage(StageParams S, int np) {
     __shared__ int64_t sh64[32];
+    __shared__ int wsum[kStageWarps];
     extern __shared__ __align__(16) unsigned char stage_smem[];
     const int inst = blockIdx.x;
     const int64_t base = S.off[inst];
@@ -117,12 +181,15 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
     // instance before anything is written: it is staged as empty with status INVAL
     const bool oob = base < 0 || n64 < 0 || n64 > S.max_n || base + n64 > S.max_total;
     const int n = oob ? 0 : int(n64);
-    int64_t bad_inval = oob ? 1 : 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0;
+    int64_t bad_inval = oob ? 1 : 0, bad_inf = 0, sum_a = 0, sum_o = 0, lmax = 0, kmax = 0, amax = 0;
     const bool in_smem = n <= np;
-    uint64_t *sk = reinterpret_cast<uint64_t *>(stage_smem);
-    int32_t *si = reinterpret_cast<int32_t *>(stage_smem + size_t(np) * 8);
-    int32_t *ss = si + np;
+    int32_t *kk = reinterpret_cast<int32_t *>(stage_smem);
+    int32_t *ka = kk + np;
+    int32_t *ss = ka + np;
     int32_t *so = ss + np;
+    int32_t *i0 = so + np;
+    int32_t *i1 = i0 + np;
+    uint16_t *cnt = reinterpret_cast<uint16_t *>(i1 + np);
     for (int j = threadIdx.x; j < n; j += blockDim.x) {
         const int64_t g = base + j;
         const int a = S.a[g], s = S.s[g], l = S.l[g], u = S.u[g], o = S.o[g];
@@ -143,10 +210,11 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
             S.lu[g] = make_int2(l, u);  // indexed by request: j == idx below
         }
         if (in_smem) {
-            sk[j] = (uint64_t(uint32_t(a)) << 32) | uint32_t(key);
-            si[j] = j;
+            kk[j] = key;
+            ka[j] = a;
             ss[j] = s;
             so[j] = o;
+            i0[j] = j;
         } else {
             QEnt e;
             e.key = key;
@@ -159,12 +227,18 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
         sum_a += a;
         sum_o += o;
         lmax = max(lmax, int64_t(max(u, o)));
+        kmax = max(kmax, int64_t(key));
+        amax = max(amax, int64_t(a));
     }
     bad_inval = block_reduce<int64_t>(bad_inval, sh64, true);
     bad_inf = block_reduce<int64_t>(bad_inf, sh64, true);
     sum_a = block_reduce<int64_t>(sum_a, sh64, false);
     sum_o = block_reduce<int64_t>(sum_o, sh64, false);
     lmax = block_reduce<int64_t>(lmax, sh64, true);
+    if (in_smem) {
+        kmax = block_reduce<int64_t>(kmax, sh64, true);
+        amax = block_reduce<int64_t>(amax, sh64, true);
+    }
     int status = ST_OK;
     if (bad_inval) status = ST_INVAL;
     else if (bad_inf) status = ST_INFEASIBLE;
@@ -184,18 +258,18 @@ __global__ void __launch_bounds__(256) k_stage(StageParams S, int np) {
         if (status == ST_OK && n > 1) bitonic_sort(S.rec + base, S.rec_a + base, n);
         return;
     }
-    if (status == ST_OK && n > 1) bitonic_sort_pairs(sk, si, n);
+    const int32_t *ord = i0;
+    if (status == ST_OK && n > 1) ord = radix_sort_idx(kk, ka, i0, i1, cnt, wsum, n, int(kmax), int(amax));
     // write the (sorted, or for a rejected instance unsorted) records out
     for (int j = threadIdx.x; j < n; j += blockDim.x) {
-        const uint64_t k = sk[j];
-        const int idx = si[j];
+        const int idx = ord[j];
         QEnt e;
-        e.key = int(uint32_t(k));
+        e.key = kk[idx];
         e.idx = idx;
         e.s = ss[idx];
         e.o = so[idx];
         S.rec[base + j] = e;
-        S.rec_a[base + j] = int(uint32_t(k >> 32));
+        S.rec_a[base + j] = ka[idx];
     }
 }
 
@@ -253,8 +327,12 @@ cudaError_t launch_stage(const StageParams &p, cudaStream_t st) {
     int np = 1;
     const int want = (p.n_max > 0 && p.n_max < kStageSmemN) ? p.n_max : kStageSmemN;
     while (np < want) np <<= 1;
-    const size_t smem = size_t(np) * kStageSmemBytesPerReq;
-    k_stage<<<p.n_inst, 256, smem, st>>>(p, np);
+    const size_t smem = size_t(np) * kStageSmemBytesPerReq + kStageCntBytes;
+    if (smem > 48 * 1024) {
+        const cudaError_t e = cudaFuncSetAttribute(k_stage, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (e != cudaSuccess) return e;
+    }
+    k_stage<<<p.n_inst, kStageThreads, smem, st>>>(p, np);
     return cudaGetLastError();
 }
 
