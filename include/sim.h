@@ -305,7 +305,7 @@ int64_t sim_kernel_launches(const sim_ctx *ctx);
  * sim_run, which sizes its launch to the whole GPU.  All calls share that array and it keeps the last call's contents: calls
  * that overlap on the GPU (different streams or threads) race; calls on one stream are safe.
  * The first call on each device looks up the array's device address (cudaGetSymbolAddress) with
- * that device current; make that first call before any stream capture.  Allocates nothing.
+ * that device current.  Allocates nothing.
  * Returns SIM_OK, SIM_E_INVAL, SIM_E_CUDA or SIM_E_STATE.
  */
 int sim_run_noalloc(int policy, int64_t M, int32_t n_instances, const int64_t *offsets, const int32_t *arrival_t,
