@@ -90,6 +90,39 @@ def _random_mixed_workload(seed, M):
     return W.concat_instances("mixed", M, parts)
 
 
+def _staging_workload(seed):
+    """Instances sized around the staging sort's boundaries (radix passes take 256 elements per
+    round, shared memory holds up to 2048 requests, larger ones go to the global-memory sort), with
+    arrival steps in random order over a wide range (several arrival-digit passes) and keys drawn
+    from a few values (long runs of ties, which the sort must keep in index order)."""
+    from fractions import Fraction
+
+    from paper_2508_14544_gb300 import workloads as W
+    rng = np.random.default_rng(seed)
+    parts = []
+    for i, n in enumerate([2, 3, 255, 256, 257, 511, 2047, 2048, 2049]):
+        s = rng.integers(1, 9, n)
+        o = rng.choice([1, 2, 3, 17, 40], n)
+        l, u = W.interval_for(o, [Fraction(1, 3), Fraction(1)][i % 2], rng)
+        if i % 3 == 0:
+            a = np.zeros(n, np.int64)
+        elif i % 3 == 1:
+            a = rng.integers(0, 1 << 20, n)  # unsorted, up to 20 bits
+        else:
+            a = rng.choice([0, 5, 4096, 70000], n)  # few distinct arrival steps
+        parts.append(dict(a=a, s=s, l=l, u=u, o=o))
+    return W.concat_instances("staging", 400, parts)
+
+
+@pytest.mark.parametrize("pol", POLS)
+def test_staging_sort_boundaries(pol):
+    w = _staging_workload(11)
+    got, comp = gpu_run(pol, w, completions=True)
+    ref, rcomp = oracle_run(pol, w, completions=True)
+    assert_same(got, ref, tag=f"staging pol={pol}")
+    assert np.array_equal(comp, rcomp)
+
+
 @pytest.mark.parametrize("M", [700, 6000])
 @pytest.mark.parametrize("pol", POLS)
 def test_random_mixed_sizes(pol, M):
