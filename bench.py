@@ -159,9 +159,46 @@ def cpu_baseline(w, budget_s: float = 20.0) -> dict:
         rs += int(plain.run_workload(pol, sample, n_threads=cores)["request_steps"].sum())
     dt = time.perf_counter() - t0
     cpu_s = time.process_time() - c0
-    return {"value": rs / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"every {stride}th instance ({sample.n_instances} of {w.n_instances}, all alphas) x 3 policies "
-                      f"(A_max, A_min, H-SF), oracle/plain.c with {cores} threads: {dt:.1f} s wall, {cpu_s:.1f} CPU-s"}
+    out = {"value": rs / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+           "sample": f"every {stride}th instance ({sample.n_instances} of {w.n_instances}, all alphas) x 3 policies "
+                     f"(A_max, A_min, H-SF), oracle/plain.c with {cores} threads: {dt:.1f} s wall, {cpu_s:.1f} CPU-s",
+           "cpu": _cpu_model()}
+    # the same oracle on one thread (16 instances, all alphas), and the literal Python oracle on
+    # the 50-request instance: the other two timing modes of the oracle
+    one = w.subset(range(0, w.n_instances, max(1, w.n_instances // 16)))
+    t0 = time.perf_counter()
+    rs1 = sum(int(plain.run_workload(pol, one, n_threads=1)["request_steps"].sum()) for pol in (0, 1, 2))
+    dt1 = time.perf_counter() - t0
+    out["single_thread"] = {"value": rs1 / dt1, "unit": UNIT, "sample": f"{one.n_instances} instances x 3 policies, "
+                                                                       f"oracle/plain.c on one thread: {dt1:.1f} s"}
+    from oracle import literal
+    from paper_2508_14544_gb300 import workloads as W
+    c1 = W.make_workload("c1").instance(0)
+    t0 = time.perf_counter()
+    rsl = sum(int(literal.simulate(pol, c1["M"], c1["a"], c1["s"], c1["l"], c1["u"], c1["o"])["request_steps"])
+              for pol in (0, 1, 2))
+    dtl = time.perf_counter() - t0
+    out["literal_c1"] = {"value": rsl / dtl, "unit": UNIT, "sample": f"the 50-request instance x 3 policies, "
+                                                                    f"oracle/literal.py: {dtl:.2f} s"}
+    return out
+
+
+def _cpu_model() -> str:
+    """The host CPU as /proc/cpuinfo names it (x86 model name, or Arm implementer / part)."""
+    import platform
+    try:
+        info = Path("/proc/cpuinfo").read_text().splitlines()
+    except OSError:
+        info = []
+    for key in ("model name", "CPU part"):
+        for line in info:
+            if line.startswith(key):
+                val = line.split(":", 1)[1].strip()
+                if key == "CPU part":
+                    impl = next((x.split(":", 1)[1].strip() for x in info if x.startswith("CPU implementer")), "?")
+                    return f"{platform.machine()} implementer {impl} part {val}"
+                return f"{platform.machine()} {val}"
+    return platform.machine()
 
 
 def run_reference(args) -> None:
