@@ -1,4 +1,4 @@
-// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared, instrumented, dense>.
+// Simulation kernel of the batched scheduler simulator (sm_103a): k_run<policy, shared, instrumented, layout>.
 //
 // One warp simulates one instance at a time (persistent warps pull instance ids from a work
 // queue).  Each step follows the paper's algorithms:
@@ -7,7 +7,8 @@
 //       jobs in ascending estimate order, ties broken uniformly at random by a key drawn afresh
 //       at every step (SplitMix64 of the instance's seed and the counter t * 2^32 + index, then
 //       the index), until it fits; each cancelled job's estimate becomes max(estimate, tokens
-//       generated) and it re-enters R_t in the same step;
+//       generated) and it re-enters R_t in the same step (the cancelled jobs stay in the
+//       active-set arrays, marked, until something reads those arrays: see the S2/S3 block);
 //   S5  admit the largest prefix of R_t (sorted by (key, index)) for which eq. Constraint holds at
 //       every future step (Algorithms malb / milb / off);
 //   S6  process the batch: one token per member, the step's memory sum(s + tokens) (eq.
@@ -24,7 +25,8 @@
 //                      (A_min) or promoted (A_ell) job
 //   B = s - p + 1      the job's memory at step x is B + x
 //   P = p, I = request index, K = the estimate (A_min key)
-// Derived arrays, recomputed in one warp pass whenever the set changes, relative to a time base tb:
+// Derived arrays, recomputed in one warp pass whenever the set changes (after A_min
+// cancellations: when they are next read), relative to a time base tb:
 //   SB[i] = sum_{j >= i} (B_j + tb),  SB[A] = 0                    (suffix sums)
 //   PM[h] = max_{i < h} H_i,  H_i = SB[i] + (A - i)(E_i - tb) + (E_i - tb),  PM[0] = -inf
 // V(x) = SB[lb] + (A - lb)(x - tb), lb = #{E < x}, is the projected memory of the active set at
