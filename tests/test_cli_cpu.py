@@ -24,3 +24,16 @@ def test_bench_reference_arm_json_line():
     assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+
+
+def test_bench_cpu_baseline_record():
+    """The bench's cpu_baseline record (all cores, one thread, the literal oracle on the
+    50-request instance, the host CPU) on a small sample, without a GPU."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    from paper_2508_14544_gb300 import workloads as W
+    w = W.make_workload("c2", range(0, 1024, 32))
+    d = bench.cpu_baseline(w, budget_s=0.5)
+    assert d["kind"] == "oracle" and d["value"] > 0 and d["cores"] >= 1 and d["unit"] == bench.UNIT
+    assert d["single_thread"]["value"] > 0 and d["literal_c1"]["value"] > 0
+    assert isinstance(d["cpu"], str) and d["cpu"]
