@@ -286,7 +286,9 @@ def sub_record(name: str, dev_id, stream, peaks_live: dict) -> dict:
             lms, rms, r = _time_runs(sim, stream, (w.offsets, *d_in), 3)
             rs = int(r["request_steps"].sum())
             p = {"sim_load_ms": round(lms, 3), "sim_run_ms": round(rms, 3), "request_steps": rs,
-                 "request_steps_per_s": rs / (rms / 1000.0)}
+                 "request_steps_per_s": rs / (rms / 1000.0),
+                 "steps_per_s": int(r["steps"].sum()) / (rms / 1000.0),
+                 "us_per_instance": round(rms * 1000.0 / w.n_instances, 3)}
             if name == "c5":
                 sim.set_option("count_work", 1)
                 r2 = sim.run(stream.cuda_stream)
