@@ -87,7 +87,10 @@ enum {
                                        (status SIM_E_STEPCAP).  0 (default): 64 * (n + sum_i o_i). */
     SIM_OPT_RECORD_COMPLETIONS = 2, /* 0/1: keep each request's completion step for
                                        sim_get_completions (default 0). */
-    SIM_OPT_WARPS_PER_BLOCK = 3,    /* 1..8: simulation warps per thread block (default 4). */
+    SIM_OPT_WARPS_PER_BLOCK = 3,    /* 1..8: simulation warps per thread block (default 4; unset,
+                                       a launch with no more instances than SMs uses 1, so that
+                                       each instance has an SM to itself).  Results do not depend
+                                       on it. */
     SIM_OPT_SMEM_ACTIVE_CAP = 4,    /* 128..4096, multiple of 128: active-set slots kept in shared
                                        memory per instance (default 512).  Instances that need more
                                        are re-run automatically with the active set in global
