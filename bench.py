@@ -266,9 +266,9 @@ def algorithmic_work(res, wc, n_requests: int) -> dict:
 
 
 def sub_record(name: str, dev_id, stream, peaks_live: dict) -> dict:
-    """One of the other configurations: per policy sim_load and sim_run device time (median of 3
-    after a warm-up), request-steps/s, the dominant kernel; on the 10^5-request workload also the
-    global-memory rate of the per-step method's queue traffic."""
+    """One of the other configurations: per policy sim_load and sim_run device time (median of 10
+    after two warm-ups), request-steps/s, steps/s, time per instance, the dominant kernel; on the
+    10^5-request workload also the global-memory rate of the per-step method's queue traffic."""
     import torch
 
     from paper_2508_14544_gb300 import SIM_AMAX, SIM_AMIN, SIM_HSF, Simulator
@@ -283,7 +283,8 @@ def sub_record(name: str, dev_id, stream, peaks_live: dict) -> dict:
             sim.load(w.offsets, *d_in)
             r = sim.run(stream.cuda_stream)  # warm-up (and residency tuning)
             assert np.all(r["status"] == 0), (name, pname, int(r["status"].min()))
-            lms, rms, r = _time_runs(sim, stream, (w.offsets, *d_in), 3)
+            sim.run(stream.cuda_stream)  # second warm-up
+            lms, rms, r = _time_runs(sim, stream, (w.offsets, *d_in), 10)
             rs = int(r["request_steps"].sum())
             p = {"sim_load_ms": round(lms, 3), "sim_run_ms": round(rms, 3), "request_steps": rs,
                  "request_steps_per_s": rs / (rms / 1000.0),
